@@ -1,0 +1,369 @@
+"""Benchmark: candidates screened per second (V filter + P score + top-k) on
+GB300, with roofline, CPU-oracle baseline and end-to-end figures.
+
+One step = one mlt_screen call over one batch of the "GEMM-style schedule
+space" workload: 65,536 candidates x 64 fp32 features, V = 200 trees of
+depth 8, P = 400 trees of depth 8, validity threshold 0.5, top-128 (the
+batch shape of ML^2Tuner's explorer step, Sec. 2; tree ensembles as in
+Table 3).  The inputs sit in HBM before the timed region; L2 is flushed
+(a 256 MB device write) before every timed step, outside its events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank screens its own batch (different seed): weak
+scaling, no collective on the data path; rank 0 prints the JSON line with
+the max-over-ranks time.  `--impl reference` times the CPU oracle instead
+(rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "candidates screened/sec (V filter + P score + top-k) at 1 GB300; % HBM roofline"
+DEFAULT_CONFIG = 2
+L2_FLUSH_BYTES = 256 << 20
+SM_COUNT = 152
+SM_MAX_MHZ_NOMINAL = 2070.0
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p.get("sm_max_mhz", SM_MAX_MHZ_NOMINAL)), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, SM_MAX_MHZ_NOMINAL, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        time.sleep(0.3)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        rows = [l.split(", ") for l in self.lines if l.count(",") >= 9]
+        mine = [r for r in rows if self.uuid and r[1].strip() == self.uuid] or rows
+        sm = [float(r[2]) for r in mine if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in mine if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in mine for i in range(4) if r[6 + i].strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(mine)}
+
+
+# ---------------------------------------------------------------------------
+# the oracle on the host cores
+# ---------------------------------------------------------------------------
+def oracle_rate(w, budget_s: float, rows_per_call: int | None = None):
+    """Single-threaded oracle throughput (candidates/s) on leading rows of
+    the workload: whole oracle passes (screen + top-k) of `rows_per_call`
+    rows until `budget_s` seconds have been spent."""
+    import oracle as O
+
+    n = w.n if rows_per_call is None else min(w.n, rows_per_call)
+    done, t0 = 0, time.perf_counter()
+    calls = 0
+    while True:
+        O.screen(w.feats[:n], w.v, w.p, w.thr, w.k)
+        done += n
+        calls += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    return done / el, {"rows_per_call": n, "calls": calls, "seconds": round(el, 3)}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2411_10764_gb300 import workloads as W
+
+    w = W.make_workload(args.config, seed=args.seed)
+    import oracle as O
+
+    O.build()
+    # size one step so that warmup + steps stay near 60 s of oracle work
+    t0 = time.perf_counter()
+    O.screen(w.feats[:1024], w.v, w.p, w.thr, w.k)
+    per_row = (time.perf_counter() - t0) / 1024
+    rows = int(max(64, min(w.n, 60.0 / max(1, args.steps + args.warmup) / max(per_row, 1e-9))))
+    for _ in range(args.warmup):
+        O.screen(w.feats[:rows], w.v, w.p, w.thr, w.k)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        O.screen(w.feats[:rows], w.v, w.p, w.thr, w.k)
+        times.append(time.perf_counter() - t0)
+    mean = sum(times) / len(times)
+    value = rows / mean
+    sample = f"first {rows} of {w.n} candidates per step (whole oracle pass: V, P, sort)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "candidates/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": mean * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config_dict(w),
+        "cpu_baseline": {"value": value, "unit": "candidates/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "candidates/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_dict(w):
+    c = w.cfg
+    return {"workload": f"{c.name} (config {c.id})", "n": w.n, "F": c.F,
+            "v_trees": c.v_trees, "v_depth": c.v_depth, "p_trees": c.p_trees, "p_depth": c.p_depth,
+            "thr": c.thr, "k": c.k, "seed": None,
+            "l2": "flushed before every timed step (256 MB device write, outside the step events)"}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def algorithmic_counts(w, survivors):
+    """Node visits and algorithmic HBM bytes of one step (see the design notes)."""
+    c = w.cfg
+    v_visits = w.n * c.v_trees * c.v_depth
+    p_visits = survivors * c.p_trees * c.p_depth
+    feat_bytes = 0 if w.feats is None else w.feats.nbytes
+    v_table = c.v_trees * (((1 << c.v_depth) - 1) * 8 + (1 << c.v_depth) * 4)
+    p_table = c.p_trees * (((1 << c.p_depth) - 1) * 8 + (1 << c.p_depth) * 4)
+    out_bytes = w.n * 8 + c.k * 8
+    return {"v_visits": v_visits, "p_visits": p_visits, "feat_bytes": feat_bytes,
+            "v_table_bytes": v_table, "p_table_bytes": p_table, "out_bytes": out_bytes,
+            "survivor_feat_bytes": survivors * c.F * 4}
+
+
+def run_ours(args):
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+
+    from paper_2411_10764_gb300 import mlt
+    from paper_2411_10764_gb300 import workloads as W
+
+    seed = args.seed + rank
+    w = W.make_workload(args.config, seed=seed)
+    mlt.load_workload_models(w)
+    x = torch.from_numpy(w.feats).to(dev)
+    n, k, thr = w.n, w.k, w.thr
+    pv = torch.empty(n, dtype=torch.float32, device=dev)
+    pf = torch.empty(n, dtype=torch.float32, device=dev)
+    tk = torch.empty(k, dtype=torch.int64, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        mlt.screen(x, thr, k, pv, pf, tk, stream=stream)
+
+    for _ in range(max(3, args.warmup)):
+        flush.fill_(1.0)
+        step()
+    mlt.sync_status(stream)
+    survivors = mlt.last_survivor_count(stream)
+
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid) if rank == 0 else None
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    if sampler:
+        sampler.start()
+    launches0 = mlt.kernel_launches()
+    mlt.profile_phases(True)
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - wall0
+    if dist is not None:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    launches = mlt.kernel_launches() - launches0
+    phases, calls = mlt.phase_times()
+    mlt.profile_phases(False)
+    mlt.sync_status(stream)
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = float(sum(step_ms))
+    if dist is not None:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * n / (ms_per_step / 1e3)
+
+    # end to end through the host-buffer entry point (pinned host memory)
+    hx = torch.from_numpy(w.feats).pin_memory()
+    hpv = torch.empty(n, dtype=torch.float32).pin_memory()
+    hpf = torch.empty(n, dtype=torch.float32).pin_memory()
+    htk = torch.empty(k, dtype=torch.int64).pin_memory()
+    out = (hpv.numpy(), hpf.numpy(), htk.numpy())
+    hxn = hx.numpy()
+    for _ in range(3):
+        mlt.screen_host(hxn, thr, k, out=out, stream=stream)
+    e2e_steps = max(10, min(args.steps, 200))
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        mlt.screen_host(hxn, thr, k, out=out, stream=stream)
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if dist is not None:
+        t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    hbm_gbs, sm_max, peak_src = peaks()
+    cnt = algorithmic_counts(w, survivors)
+    v_ms = phases["v_pass"] / max(calls, 1)
+    p_ms = phases["p_pass"] / max(calls, 1)
+    dominant = "v_pass" if v_ms >= p_ms else "p_pass"
+    dom_ms = max(v_ms, p_ms)
+    dom_visits = cnt["v_visits"] if dominant == "v_pass" else cnt["p_visits"]
+    # one shared-memory gather of x[feature] per node visit, 32 lanes per
+    # clock per SM: the on-chip issue ceiling of the walk
+    visit_peak = SM_COUNT * 32 * sm_max * 1e6
+    achieved = dom_visits / (dom_ms / 1e3)
+    dom_bytes = (cnt["feat_bytes"] + cnt["v_table_bytes"]) if dominant == "v_pass" else \
+        (cnt["survivor_feat_bytes"] + cnt["p_table_bytes"])
+    step_bytes = cnt["feat_bytes"] + cnt["v_table_bytes"] + cnt["p_table_bytes"]
+    traffic = None
+    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tr_path):
+        try:
+            with open(tr_path) as f:
+                tr = json.load(f)
+            ent = tr.get(f"config{args.config}:{dominant}")
+            traffic = ent.get("dram_bytes_per_launch") if ent else None
+        except (OSError, ValueError):
+            traffic = None
+    line = {
+        "metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded; shapes of the paper's tuning tasks)",
+        "config": dict(config_dict(w), seed=args.seed, parallelism=f"replicas x{world}"),
+        "survivors": survivors,
+        "phases_ms": {kk: vv / max(calls, 1) for kk, vv in phases.items()},
+        "roofline": {
+            "bound": "alu", "kernel": f"{dominant} (tree walk)",
+            "achieved": achieved / 1e9, "peak": visit_peak / 1e9, "unit": "Gvisit/s",
+            "frac": achieved / visit_peak, "traffic": traffic,
+            "peak_note": f"152 SMs x 32 shared-memory lanes/clk x {sm_max:.0f} MHz: one x[f] gather per node visit",
+        },
+        "hbm_roofline": {
+            "bound": "hbm", "achieved": step_bytes / (ms_per_step / 1e3) / 1e9, "peak": hbm_gbs,
+            "unit": "GB/s", "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / hbm_gbs,
+            "peak_source": peak_src, "bytes_per_step": step_bytes,
+            "dominant_kernel_gbs": dom_bytes / (dom_ms / 1e3) / 1e9,
+        },
+        "e2e": {"value": world * n / e2e_s, "unit": "candidates/s",
+                "h2d_bytes_per_step": int(w.feats.nbytes),
+                "d2h_bytes_per_step": int(2 * n * 4 + k * 8)},
+        "gpu_launches": int(launches),
+        "clocks": clocks,
+        "wall_ms_per_step_incl_flush": wall * 1e3 / args.steps,
+    }
+    if not args.no_cpu_baseline:
+        rate, info = oracle_rate(w, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": rate, "unit": "candidates/s", "cores": 1, "kind": "oracle",
+                                "sample": f"whole workload ({info['rows_per_call']} candidates) x "
+                                          f"{info['calls']} oracle passes, {info['seconds']} s, single thread"}
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=DEFAULT_CONFIG)
+    ap.add_argument("--seed", type=int, default=1)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,207 @@
+/*
+ * mlt.h -- C ABI of libmlt, GB300 (sm_103a) batched candidate screening for
+ * ML^2Tuner-style autotuning (arXiv 2411.10764).
+ *
+ * The paper's configuration explorer scores candidate code configurations
+ * with a validity model V and a performance model P, drops the candidates V
+ * predicts invalid, and keeps the (alpha+1)N candidates that P ranks best
+ * (Sec. 2, "Configuration Explorer", "ML Model V", "ML Model P", "Hidden
+ * Feature Extractor & ML Model A").  All models are XGBoost tree ensembles
+ * (Sec. 3 "Experimental Setup"; Appendix A.3, Table 3).  This library runs
+ * that inner step over a whole batch of candidates on one GPU.
+ *
+ * Conventions for every call:
+ *   - Every function returns an mlt_status (0 = MLT_OK, negative = error)
+ *     and never aborts or traps.  mlt_last_error() gives a message for the
+ *     last failing call on the calling thread.
+ *   - "device" pointers are CUDA device memory owned by the caller (for
+ *     example torch tensors); "host" pointers are ordinary host memory.
+ *     The library keeps no reference to a caller buffer after the call (or,
+ *     for asynchronous calls, after the queued GPU work has finished).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Asynchronous calls only enqueue work on it; errors detected
+ *     by the GPU (a bounded wait that gave up) are reported by the next
+ *     mlt_sync_status() on that stream.
+ *   - Library state (loaded ensembles, feature count, scratch buffers) is
+ *     process-wide and guarded by a lock; scratch buffers are shared, so
+ *     screening calls must be ordered on one stream (or the caller must
+ *     synchronize between streams).
+ *   - Candidate counts are limited to n < 2^31; top-k to 1 <= k <= 16384.
+ */
+#ifndef MLT_H
+#define MLT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MLT_OK = 0,
+    MLT_EINVAL = -1,   /* bad argument or malformed ensemble / program     */
+    MLT_ENOMODEL = -2, /* screening asked for a model that is not loaded   */
+    MLT_ECUDA = -3,    /* a CUDA runtime call failed (message has details) */
+    MLT_ENOMEM = -4,   /* device or host allocation failed                 */
+    MLT_ETIMEOUT = -5  /* a bounded device-side wait gave up               */
+} mlt_status;
+
+/* Model slots (Sec. 2): V = validity classifier, P = performance regressor,
+ * A = the hidden-feature performance model used to rerank the kept set. */
+enum { MLT_MODEL_V = 0, MLT_MODEL_P = 1, MLT_MODEL_A = 2 };
+
+/* One tree slot in implicit heap order (12 bytes).  A tree of depth d has
+ * 2^(d+1)-1 slots; the children of slot j are 2j+1 (left) and 2j+2 (right).
+ *   feature >= 0 : split; x[feature] < value goes left, x >= value goes
+ *                  right, a NaN (missing) x goes left iff default_left != 0;
+ *   feature == -1: leaf with output `value`;
+ *   feature == -2: unused slot (below a leaf, or past the tree's depth).
+ * This is XGBoost's gbtree routing rule (Sec. 3 setup, Table 3); the paper
+ * does not spell out the comparison, the strict `<` is this library's
+ * reading. */
+typedef struct {
+    int32_t feature;
+    float value;
+    uint8_t default_left;
+    uint8_t pad[3];
+} mlt_node;
+
+/* One instruction of a feature program (16 bytes); see mlt_decode_knobs. */
+typedef struct {
+    int32_t op;
+    int32_t a;
+    int32_t b;
+    float c;
+} mlt_feat_op;
+
+/* Feature-program opcodes.  Operands a, b: -1 = the constant c; 0..K-1 =
+ * knob j's option value; K+f = feature f of the same candidate, f below the
+ * feature being computed.  Every operation is one IEEE-754 binary32
+ * operation rounded to nearest (no fused multiply-add). */
+enum {
+    MLT_OP_COPY = 0,    /* A                                               */
+    MLT_OP_ILOG2 = 1,   /* floor(log2 A) for a positive normal A, else 0    */
+    MLT_OP_ADD = 2,     /* A + B                                           */
+    MLT_OP_SUB = 3,     /* A - B                                           */
+    MLT_OP_MUL = 4,     /* A * B                                           */
+    MLT_OP_DIV = 5,     /* A / B                                           */
+    MLT_OP_CEILDIV = 6, /* ceil(A / B)                                     */
+    MLT_OP_REM = 7,     /* A - B * floor(A / B), three rounded operations  */
+    MLT_OP_MIN = 8,     /* (B < A) ? B : A                                 */
+    MLT_OP_MAX = 9,     /* (B > A) ? B : A                                 */
+    MLT_OP_GT = 10,     /* (A > B) ? 1 : 0                                 */
+    MLT_OP_EQ = 11      /* (A == B) ? 1 : 0                                */
+};
+
+/* Number of features F per candidate (1 <= F <= 1024).  Must be set before
+ * loading ensembles; changing it unloads every ensemble.  Synchronous. */
+int mlt_set_num_features(int F);
+
+/* Copy, validate and pack one ensemble into library-owned device memory
+ * (Sec. 2: model V, P or A; Table 3: XGBoost gbtree).
+ *   model_id : MLT_MODEL_V, MLT_MODEL_P or MLT_MODEL_A
+ *   nodes    : host array of n_trees * (2^(depth+1)-1) heap-order slots;
+ *              the caller keeps ownership (it is only read during the call)
+ *   n_trees  : 1 .. 65536;  depth : 1 .. 12
+ * Validation (MLT_EINVAL): slot 0 is a split or a leaf; every split's two
+ * children are splits or leaves; slots at `depth` that are reachable are
+ * leaves; split features lie in [0, F); thresholds and leaves are finite;
+ * the sum over trees of the largest |leaf| is below 1e37 (no fp32 overflow
+ * in the leaf sum).  Replaces a previously loaded model in the same slot.
+ * Synchronous (waits for queued work before freeing an old table). */
+int mlt_load_ensemble(int model_id, const mlt_node *nodes, int n_trees, int depth);
+
+/* Free a loaded ensemble (no-op if the slot is empty).  Synchronous. */
+int mlt_free_ensemble(int model_id);
+
+/* The validity cut in margin space: *tau_out = the smallest float m with
+ * sigmoid(m) >= thr, 0 < thr < 1 (thr = 0.5 gives 0, the sign rule of the
+ * paper's binary:hinge model V, Table 3).  A candidate is valid iff its V
+ * margin >= tau.  Host-only. */
+int mlt_validity_cut(float thr, float *tau_out);
+
+/* Screen a batch of candidates (the explorer's inner step, Sec. 2):
+ *   margin_V(i) = sum over V's trees of the leaf row i reaches, fp32, in
+ *                 tree order from 0.0f;  valid(i) = margin_V(i) >= tau(thr)
+ *   out_pvalid[i] = sigmoid(margin_V(i))                       (fp32)
+ *   out_perf[i]   = margin_P(i) if valid(i), else -infinity     (fp32)
+ *   out_topk[r]   = index of the r-th best valid candidate by
+ *                   (margin_P descending, index ascending), r < k;
+ *                   -1 where fewer than k candidates are valid.
+ * Arguments:
+ *   feats      device, row-major [n][F] fp32 (NaN = missing value)
+ *   n          0 .. 2^31-1 candidates;  thr in (0, 1);  k in 1 .. 16384
+ *   out_pvalid device [n] fp32;  out_perf device [n] fp32
+ *   out_topk   device [k] int64
+ * Needs models V and P loaded with the current F (MLT_ENOMODEL otherwise).
+ * Asynchronous on `stream`; uses library scratch sized by n (allocated on
+ * first use or growth). */
+int mlt_screen(void *stream, const float *feats, int64_t n, float thr, int k,
+               float *out_pvalid, float *out_perf, int64_t *out_topk);
+
+/* mlt_screen with host buffers, for end-to-end use: copies feats_host
+ * ([n][F] fp32) to the device, screens, and copies the three results back
+ * into host buffers of the same shapes.  Synchronous on `stream`. */
+int mlt_screen_host(void *stream, const float *feats_host, int64_t n, float thr, int k,
+                    float *pvalid_host, float *perf_host, int64_t *topk_host);
+
+/* Decode candidate indices into knob choices and build their features
+ * (the explorer's enumeration of the search space, Sec. 2; knobs are tiling
+ * sizes and virtual-thread counts, Appendix A.2; derived features after
+ * Table 5).  Candidate i (first_index <= i < first_index + n) is the
+ * mixed-radix number with digit j = floor(i / prod_{l<j} r_l) mod r_j, knob
+ * 0 least significant; knob j takes option_values[off_j + digit_j] with
+ * off_j = r_0 + ... + r_{j-1}.  Feature f is program[f] evaluated on the
+ * knob values and the features before it.
+ *   radices       host [n_knobs], each 1 .. 256;  n_knobs 1 .. 16;
+ *                 sum of radices <= 256
+ *   option_values host, the concatenated option tables
+ *   program       host [F] instructions, 1 <= F <= 256
+ *   first_index + n <= product of the radices
+ *   out_knobs     device [n][n_knobs] uint8 option indices, or NULL
+ *   out_feats     device [n][F] fp32, or NULL
+ * Asynchronous on `stream`. */
+int mlt_decode_knobs(void *stream, const int32_t *radices, const float *option_values,
+                     int n_knobs, const mlt_feat_op *program, int F, int64_t first_index,
+                     int64_t n, uint8_t *out_knobs, float *out_feats);
+
+/* mlt_screen over decoded candidates first_index .. first_index+n-1: the
+ * features are built on chip inside the screening kernels and never stored.
+ * The program length must equal the current F.  out_topk holds candidate
+ * indices (first_index + position).  Asynchronous on `stream`. */
+int mlt_screen_decoded(void *stream, const int32_t *radices, const float *option_values,
+                       int n_knobs, const mlt_feat_op *program, int64_t first_index,
+                       int64_t n, float thr, int k, float *out_pvalid, float *out_perf,
+                       int64_t *out_topk);
+
+/* Wait for `stream` and report errors its queued library work met on the
+ * device (MLT_ETIMEOUT for a bounded wait that gave up), clearing them. */
+int mlt_sync_status(void *stream);
+
+/* Number of valid candidates found by the last screening call (waits for
+ * `stream`). */
+int mlt_last_survivor_count(void *stream, int64_t *count_out);
+
+/* Measurement support.  mlt_profile_phases(1) makes every later screening
+ * call record CUDA events between its phases on the caller's stream (and
+ * clears earlier records); mlt_profile_phases(0) stops recording.  Host-only
+ * bookkeeping plus event records; results are unchanged. */
+int mlt_profile_phases(int enable);
+
+/* Waits for the recorded events, then writes for each phase the device time
+ * summed over the recorded calls, in ms: out_ms[0] V pass, [1] survivor
+ * compaction, [2] P pass, [3] top-k (n_phases <= 4 entries written).
+ * *n_calls_out receives the number of recorded calls.  Clears the records. */
+int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
+
+/* Cumulative number of GPU kernels this library has launched. */
+int64_t mlt_kernel_launches(void);
+
+/* Message for the last failing call on this thread ("" if none). */
+const char *mlt_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MLT_H */

@@ -1,0 +1,645 @@
+// libmlt C ABI: argument validation, ensemble packing, scratch management
+// and the launch sequence of one screening pass (see include/mlt.h).
+//
+// ML^2Tuner (arXiv 2411.10764) Sec. 2: the explorer applies model V and
+// model P to candidate configurations, discards those V predicts invalid and
+// keeps the (alpha+1)N best by P.  One mlt_screen call = that step over a
+// whole batch:
+//   V pass (traverse.cu)  -> validity ballots, pvalid, -inf for the invalid
+//   compaction (select.cu) -> ascending survivor list
+//   P pass (traverse.cu)  -> P score per survivor + 64-bit rank keys
+//   radix select + sort (select.cu) -> top-k indices
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "mlt.h"
+#include "mlt_internal.cuh"
+
+namespace {
+
+using namespace mlt;
+
+thread_local std::string t_err;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  t_err = buf;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(MLT_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define MLT_CUDA(call, what)                      \
+  do {                                            \
+    cudaError_t e_ = (call);                      \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+struct Model {
+  bool loaded = false;
+  int device = -1;
+  int F = 0;
+  DeviceModel dm;
+  unsigned char* owned = nullptr;
+};
+
+struct ScratchOwner {
+  int device = -1;
+  long long cap_n = -1;  // capacity in candidates
+  Scratch s;
+  void* block = nullptr;  // one allocation for everything sized by n
+  SelectState* state = nullptr;
+  unsigned long long* sel = nullptr;
+  unsigned int* err = nullptr;
+  // host-buffer entry point staging
+  long long host_cap_n = -1;
+  int host_cap_F = 0;
+  float* h_feats = nullptr;
+  float* h_pvalid = nullptr;
+  float* h_perf = nullptr;
+  int64_t* h_topk = nullptr;
+};
+
+std::mutex g_mu;
+int g_F = 0;
+long long g_launches = 0;
+
+// Phase profiling: one set of 5 events per recorded screening call.
+constexpr int kPhases = 4;
+bool g_profile = false;
+std::vector<cudaEvent_t> g_events;  // pool, 5 per call
+size_t g_events_used = 0;
+Model g_models[3];
+ScratchOwner g_scr;
+int g_optin = -1;
+
+size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
+
+int current_device(int* dev) {
+  MLT_CUDA(cudaGetDevice(dev), "cudaGetDevice");
+  return MLT_OK;
+}
+
+int smem_optin() {
+  if (g_optin < 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 48 * 1024;
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+      return 48 * 1024;
+    g_optin = v;
+  }
+  return g_optin;
+}
+
+void free_model(Model& m) {
+  if (m.owned != nullptr) {
+    cudaDeviceSynchronize();  // queued screens may still read the table
+    cudaFree(m.owned);
+  }
+  m = Model();
+}
+
+// Scratch sized by n candidates (plus the fixed pieces).
+int ensure_scratch(long long n) {
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  if (g_scr.err == nullptr || g_scr.device != dev) {
+    if (g_scr.device != -1 && g_scr.device != dev)
+      return fail(MLT_EINVAL, "libmlt scratch lives on device %d, current device is %d", g_scr.device, dev);
+    MLT_CUDA(cudaMalloc(&g_scr.err, sizeof(unsigned int)), "cudaMalloc(error word)");
+    MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(unsigned int)), "cudaMemset(error word)");
+    MLT_CUDA(cudaMalloc(&g_scr.state, sizeof(SelectState)), "cudaMalloc(select state)");
+    MLT_CUDA(cudaMemset(g_scr.state, 0, sizeof(SelectState)), "cudaMemset(select state)");
+    MLT_CUDA(cudaMalloc(&g_scr.sel, sizeof(unsigned long long) * kMaxK), "cudaMalloc(selection)");
+    g_scr.device = dev;
+  }
+  if (n > g_scr.cap_n) {
+    long long cap = n < 1024 ? 1024 : n;
+    const long long words = (cap + 31) / 32 + 8;
+    const size_t b_masks = align16(words * 4);
+    const size_t b_tiles = align16(words * 4);  // tiles are >= 32 candidates
+    const size_t b_rows = align16(cap * 4);
+    const size_t b_keys = align16(cap * 8);
+    const size_t total = b_masks + 2 * b_tiles + b_rows + b_keys;
+    if (g_scr.block != nullptr) {
+      cudaDeviceSynchronize();
+      cudaFree(g_scr.block);
+      g_scr.block = nullptr;
+      g_scr.cap_n = -1;
+    }
+    void* blk = nullptr;
+    cudaError_t e = cudaMalloc(&blk, total);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(MLT_ENOMEM, "cannot allocate %zu bytes of screening scratch", total);
+    }
+    unsigned char* p = static_cast<unsigned char*>(blk);
+    g_scr.s.masks = reinterpret_cast<uint32_t*>(p);
+    p += b_masks;
+    g_scr.s.tile_counts = reinterpret_cast<uint32_t*>(p);
+    p += b_tiles;
+    g_scr.s.tile_offsets = reinterpret_cast<uint32_t*>(p);
+    p += b_tiles;
+    g_scr.s.rows = reinterpret_cast<uint32_t*>(p);
+    p += b_rows;
+    g_scr.s.keys = reinterpret_cast<unsigned long long*>(p);
+    g_scr.block = blk;
+    g_scr.cap_n = cap;
+  }
+  g_scr.s.state = g_scr.state;
+  g_scr.s.sel = g_scr.sel;
+  g_scr.s.err = g_scr.err;
+  return MLT_OK;
+}
+
+// sigmoid(m) >= thr  <=>  thr * (1 + e^-m) <= 1  <=>  thr * expm1(-m) <= 1 - 2 thr
+bool cut_passes(float m, float thr) {
+  const long double lhs = static_cast<long double>(thr) * expm1l(-static_cast<long double>(m));
+  const long double rhs = 1.0L - 2.0L * static_cast<long double>(thr);
+  return lhs <= rhs;
+}
+
+float validity_cut(float thr) {
+  float m = static_cast<float>(std::log(static_cast<double>(thr) / (1.0 - static_cast<double>(thr))));
+  if (!cut_passes(m, thr)) {
+    while (!cut_passes(m, thr)) m = std::nextafterf(m, INFINITY);
+  } else {
+    for (;;) {
+      const float d = std::nextafterf(m, -INFINITY);
+      if (!cut_passes(d, thr)) break;
+      m = d;
+    }
+  }
+  return m == 0.0f ? 0.0f : m;
+}
+
+int check_screen_args(long long n, float thr, int k) {
+  if (n < 0 || n > 0x7FFFFFFFLL) return fail(MLT_EINVAL, "n must lie in [0, 2^31-1], got %lld", n);
+  if (!(thr > 0.0f && thr < 1.0f)) return fail(MLT_EINVAL, "thr must lie in (0, 1)");
+  if (k < 1 || k > kMaxK) return fail(MLT_EINVAL, "k must lie in [1, %d], got %d", kMaxK, k);
+  return MLT_OK;
+}
+
+int check_models(int dev) {
+  for (int id : {MLT_MODEL_V, MLT_MODEL_P}) {
+    const Model& m = g_models[id];
+    if (!m.loaded) return fail(MLT_ENOMODEL, "model %s is not loaded", id == 0 ? "V" : "P");
+    if (m.F != g_F) return fail(MLT_ENOMODEL, "model %s was loaded for F=%d, current F=%d", id == 0 ? "V" : "P", m.F, g_F);
+    if (m.device != dev) return fail(MLT_EINVAL, "model %s lives on device %d, current device is %d", id == 0 ? "V" : "P", m.device, dev);
+  }
+  return MLT_OK;
+}
+
+ScreenShape plan_for(const DeviceModel& dm, int F) {
+  if (dm.kind == kTableFull) return plan_full(F, dm.depth, dm.n_trees, dm.tree_bytes, smem_optin());
+  return plan_compact(F, smem_optin());
+}
+
+int build_decoder(const int32_t* radices, const float* option_values, int n_knobs,
+                  const mlt_feat_op* program, int F, long long first_index, long long n,
+                  DecodeParams* d) {
+  if (radices == nullptr || option_values == nullptr || program == nullptr)
+    return fail(MLT_EINVAL, "radices, option_values and program must be non-NULL");
+  if (n_knobs < 1 || n_knobs > kMaxKnobs) return fail(MLT_EINVAL, "n_knobs must lie in [1, %d]", kMaxKnobs);
+  if (F < 1 || F > kMaxProgram) return fail(MLT_EINVAL, "program length must lie in [1, %d]", kMaxProgram);
+  if (first_index < 0 || n < 0) return fail(MLT_EINVAL, "first_index and n must be non-negative");
+  std::memset(d, 0, sizeof(*d));
+  d->n_knobs = n_knobs;
+  d->F = F;
+  d->first_index = first_index;
+  int off = 0;
+  long double space = 1.0L;
+  for (int j = 0; j < n_knobs; ++j) {
+    if (radices[j] < 1 || radices[j] > 256) return fail(MLT_EINVAL, "radix %d of knob %d outside [1, 256]", radices[j], j);
+    d->radix[j] = radices[j];
+    d->opt_off[j] = off;
+    off += radices[j];
+    if (off > kMaxOptions) return fail(MLT_EINVAL, "more than %d option values in total", kMaxOptions);
+    space *= radices[j];
+  }
+  if (static_cast<long double>(first_index) + static_cast<long double>(n) > space)
+    return fail(MLT_EINVAL, "candidates past the end of the knob space");
+  std::memcpy(d->opts, option_values, sizeof(float) * off);
+  for (int f = 0; f < F; ++f) {
+    const mlt_feat_op& o = program[f];
+    if (o.op < 0 || o.op > MLT_OP_EQ) return fail(MLT_EINVAL, "feature %d: unknown opcode %d", f, o.op);
+    if (o.a < -1 || o.a >= n_knobs + f || o.b < -1 || o.b >= n_knobs + f)
+      return fail(MLT_EINVAL, "feature %d: operand refers to an unknown slot", f);
+    d->op[f] = o.op;
+    d->a[f] = o.a;
+    d->b[f] = o.b;
+    d->c[f] = o.c;
+  }
+  return MLT_OK;
+}
+
+// Validate the heap-order ensemble and pack it for the device.
+int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vector<unsigned char>& out,
+                  DeviceModel& dm) {
+  const int slots = (2 << depth) - 1;
+  std::vector<unsigned char> reach(slots);
+  std::vector<int> depth_of(slots);
+  for (int j = 0; j < slots; ++j) depth_of[j] = 31 - __builtin_clz(static_cast<unsigned>(j + 1));
+  long double leaf_bound = 0.0L;
+  for (int t = 0; t < n_trees; ++t) {
+    const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+    std::fill(reach.begin(), reach.end(), 0);
+    reach[0] = 1;
+    float maxabs = 0.0f;
+    for (int j = 0; j < slots; ++j) {
+      if (!reach[j]) continue;
+      const mlt_node& nd = tr[j];
+      if (nd.feature == -2) return fail(MLT_EINVAL, "tree %d slot %d: reachable slot is unused", t, j);
+      if (nd.feature < -2) return fail(MLT_EINVAL, "tree %d slot %d: bad feature code %d", t, j, nd.feature);
+      if (!std::isfinite(nd.value)) return fail(MLT_EINVAL, "tree %d slot %d: value is not finite", t, j);
+      if (nd.feature == -1) {
+        maxabs = std::fmax(maxabs, std::fabs(nd.value));
+        continue;
+      }
+      if (depth_of[j] >= depth) return fail(MLT_EINVAL, "tree %d slot %d: split below the depth limit", t, j);
+      if (nd.feature >= F) return fail(MLT_EINVAL, "tree %d slot %d: feature %d >= F=%d", t, j, nd.feature, F);
+      reach[2 * j + 1] = 1;
+      reach[2 * j + 2] = 1;
+    }
+    leaf_bound += maxabs;
+  }
+  if (leaf_bound >= 1e37L) return fail(MLT_EINVAL, "leaf magnitudes could overflow the fp32 sum");
+
+  dm.n_trees = n_trees;
+  dm.depth = depth;
+  if (depth <= kMaxFullDepth) {
+    const uint32_t I = (1u << depth) - 1u, L = 1u << depth;
+    const size_t tb = align16(static_cast<size_t>(I) * 8 + static_cast<size_t>(L) * 4);
+    dm.kind = kTableFull;
+    dm.tree_bytes = static_cast<uint32_t>(tb);
+    out.assign(tb * n_trees, 0);
+    std::vector<float> inherit(slots);
+    for (int t = 0; t < n_trees; ++t) {
+      const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+      unsigned char* dst = out.data() + tb * t;
+      std::fill(reach.begin(), reach.end(), 0);
+      reach[0] = 1;
+      for (int j = 0; j < slots; ++j) {
+        const mlt_node& nd = tr[j];
+        const bool split = reach[j] && nd.feature >= 0;
+        if (split) {
+          reach[2 * j + 1] = 1;
+          reach[2 * j + 2] = 1;
+        }
+        if (reach[j] && nd.feature == -1)
+          inherit[j] = nd.value;
+        else if (!reach[j])
+          inherit[j] = inherit[(j - 1) / 2];  // below a leaf: copy it down
+        else
+          inherit[j] = 0.0f;
+        if (static_cast<uint32_t>(j) < I) {
+          float thr = 0.0f;
+          uint32_t meta = 0;
+          if (split) {
+            thr = nd.value;
+            meta = static_cast<uint32_t>(nd.feature) | (nd.default_left ? kMetaDefaultLeft : 0u);
+          }
+          std::memcpy(dst + 8 * j, &thr, 4);
+          std::memcpy(dst + 8 * j + 4, &meta, 4);
+        } else {
+          const float leaf = inherit[j];
+          std::memcpy(dst + 8 * I + 4 * (j - I), &leaf, 4);
+        }
+      }
+    }
+  } else {
+    dm.kind = kTableCompact;
+    dm.tree_bytes = 0;
+    std::vector<uint32_t> offsets(n_trees);
+    std::vector<uint32_t> recs;
+    std::vector<int> order;
+    for (int t = 0; t < n_trees; ++t) {
+      const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+      offsets[t] = static_cast<uint32_t>(recs.size() / 2);
+      order.assign(1, 0);
+      for (size_t q = 0; q < order.size(); ++q) {
+        const mlt_node& nd = tr[order[q]];
+        float v = nd.value;
+        uint32_t meta;
+        if (nd.feature >= 0) {
+          const uint32_t left = static_cast<uint32_t>(order.size());
+          if (left > 0x3FFFu) return fail(MLT_EINVAL, "tree %d has too many nodes", t);
+          order.push_back(2 * order[q] + 1);
+          order.push_back(2 * order[q] + 2);
+          meta = static_cast<uint32_t>(nd.feature) | (left << 16) | (nd.default_left ? kMetaDefaultLeft : 0u);
+        } else {
+          meta = kMetaLeaf;
+        }
+        uint32_t vb;
+        std::memcpy(&vb, &v, 4);
+        recs.push_back(vb);
+        recs.push_back(meta);
+      }
+    }
+    const size_t head = align16(static_cast<size_t>(n_trees) * 4);
+    out.assign(head + recs.size() * 4, 0);
+    std::memcpy(out.data(), offsets.data(), offsets.size() * 4);
+    std::memcpy(out.data() + head, recs.data(), recs.size() * 4);
+  }
+  return MLT_OK;
+}
+
+// The whole screening sequence on `st` (caller holds g_mu).
+int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, long long n, float thr,
+               int k, float* out_pvalid, float* out_perf, int64_t* out_topk) {
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  rc = check_models(dev);
+  if (rc != MLT_OK) return rc;
+  rc = ensure_scratch(n);
+  if (rc != MLT_OK) return rc;
+  const DeviceModel& V = g_models[MLT_MODEL_V].dm;
+  const DeviceModel& P = g_models[MLT_MODEL_P].dm;
+  const ScreenShape sv = plan_for(V, g_F), sp = plan_for(P, g_F);
+  if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
+  const Scratch& s = g_scr.s;
+  TraverseArgs a{};
+  a.feats = feats;
+  a.F = g_F;
+  a.n = n;
+  a.vec4 = (feats != nullptr && (reinterpret_cast<uintptr_t>(feats) & 15u) == 0 && (g_F & 3) == 0) ? 1 : 0;
+  a.state = s.state;
+  a.rows = s.rows;
+  a.tau = validity_cut(thr);
+  a.out_pvalid = out_pvalid;
+  a.out_perf = out_perf;
+  a.masks = s.masks;
+  a.tile_counts = s.tile_counts;
+  a.keys = s.keys;
+  a.err = s.err;
+  a.decode = dec != nullptr;
+
+  TraverseArgs av = a;
+  av.p_pass = 0;
+  av.table = V.table;
+  av.n_trees = V.n_trees;
+  av.tree_bytes = V.tree_bytes;
+  av.chunk_trees = sv.chunk_trees;
+  av.nbuf = sv.nbuf;
+  av.max_depth = V.depth;
+  cudaEvent_t* ev = nullptr;
+  if (g_profile) {
+    if (g_events_used + kPhases + 1 > g_events.size()) {
+      for (int i = 0; i <= kPhases; ++i) {
+        cudaEvent_t e;
+        MLT_CUDA(cudaEventCreate(&e), "cudaEventCreate");
+        g_events.push_back(e);
+      }
+    }
+    ev = &g_events[g_events_used];
+    g_events_used += kPhases + 1;
+    MLT_CUDA(cudaEventRecord(ev[0], st), "cudaEventRecord");
+  }
+  const long long tiles_v = (n + sv.threads - 1) / sv.threads;
+  MLT_CUDA(launch_traverse(V, av, dec, sv, tiles_v, st), "V pass launch");
+  if (ev) MLT_CUDA(cudaEventRecord(ev[1], st), "cudaEventRecord");
+  MLT_CUDA(launch_compact(s, n, sv.threads, tiles_v, k, st), "compaction launch");
+  if (ev) MLT_CUDA(cudaEventRecord(ev[2], st), "cudaEventRecord");
+
+  TraverseArgs ap = a;
+  ap.p_pass = 1;
+  ap.table = P.table;
+  ap.n_trees = P.n_trees;
+  ap.tree_bytes = P.tree_bytes;
+  ap.chunk_trees = sp.chunk_trees;
+  ap.nbuf = sp.nbuf;
+  ap.max_depth = P.depth;
+  const long long tiles_p = (n + sp.threads - 1) / sp.threads;
+  MLT_CUDA(launch_traverse(P, ap, dec, sp, tiles_p, st), "P pass launch");
+  if (ev) MLT_CUDA(cudaEventRecord(ev[3], st), "cudaEventRecord");
+  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, st), "top-k launch");
+  if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
+  g_launches += (tiles_v > 0 ? 1 : 0) + 1 + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + kRadixPasses + 2;
+  return MLT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int mlt_set_num_features(int F) {
+  if (F < 1 || F > kMaxF) return fail(MLT_EINVAL, "F must lie in [1, %d], got %d", kMaxF, F);
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (F != g_F)
+    for (Model& m : g_models) free_model(m);
+  g_F = F;
+  return MLT_OK;
+}
+
+int mlt_load_ensemble(int model_id, const mlt_node* nodes, int n_trees, int depth) {
+  if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
+  if (nodes == nullptr) return fail(MLT_EINVAL, "nodes must be non-NULL");
+  if (n_trees < 1 || n_trees > 65536) return fail(MLT_EINVAL, "n_trees must lie in [1, 65536], got %d", n_trees);
+  if (depth < 1 || depth > kMaxDepth) return fail(MLT_EINVAL, "depth must lie in [1, %d], got %d", kMaxDepth, depth);
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_EINVAL, "call mlt_set_num_features before loading ensembles");
+  std::vector<unsigned char> packed;
+  DeviceModel dm;
+  int rc = pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
+  if (rc != MLT_OK) return rc;
+  int dev = 0;
+  rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  unsigned char* d = nullptr;
+  cudaError_t e = cudaMalloc(&d, packed.size());
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(MLT_ENOMEM, "cannot allocate %zu bytes for the ensemble", packed.size());
+  }
+  e = cudaMemcpy(d, packed.data(), packed.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cudaFree(d);
+    return cuda_fail(e, "ensemble upload");
+  }
+  free_model(g_models[model_id]);
+  Model& m = g_models[model_id];
+  m.loaded = true;
+  m.device = dev;
+  m.F = g_F;
+  m.owned = d;
+  m.dm = dm;
+  m.dm.table = d;
+  m.dm.bytes = packed.size();
+  return MLT_OK;
+}
+
+int mlt_free_ensemble(int model_id) {
+  if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
+  std::lock_guard<std::mutex> lk(g_mu);
+  free_model(g_models[model_id]);
+  return MLT_OK;
+}
+
+int mlt_validity_cut(float thr, float* tau_out) {
+  if (tau_out == nullptr) return fail(MLT_EINVAL, "tau_out must be non-NULL");
+  if (!(thr > 0.0f && thr < 1.0f)) return fail(MLT_EINVAL, "thr must lie in (0, 1)");
+  *tau_out = validity_cut(thr);
+  return MLT_OK;
+}
+
+int mlt_screen(void* stream, const float* feats, int64_t n, float thr, int k, float* out_pvalid,
+               float* out_perf, int64_t* out_topk) {
+  int rc = check_screen_args(n, thr, k);
+  if (rc != MLT_OK) return rc;
+  if ((n > 0 && (feats == nullptr || out_pvalid == nullptr || out_perf == nullptr)) || out_topk == nullptr)
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  return run_screen(static_cast<cudaStream_t>(stream), feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk);
+}
+
+int mlt_screen_decoded(void* stream, const int32_t* radices, const float* option_values, int n_knobs,
+                       const mlt_feat_op* program, int64_t first_index, int64_t n, float thr, int k,
+                       float* out_pvalid, float* out_perf, int64_t* out_topk) {
+  int rc = check_screen_args(n, thr, k);
+  if (rc != MLT_OK) return rc;
+  if ((n > 0 && (out_pvalid == nullptr || out_perf == nullptr)) || out_topk == nullptr)
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  DecodeParams d;
+  rc = build_decoder(radices, option_values, n_knobs, program, g_F, first_index, n, &d);
+  if (rc != MLT_OK) return rc;
+  return run_screen(static_cast<cudaStream_t>(stream), nullptr, &d, n, thr, k, out_pvalid, out_perf, out_topk);
+}
+
+int mlt_screen_host(void* stream, const float* feats_host, int64_t n, float thr, int k, float* pvalid_host,
+                    float* perf_host, int64_t* topk_host) {
+  int rc = check_screen_args(n, thr, k);
+  if (rc != MLT_OK) return rc;
+  if ((n > 0 && (feats_host == nullptr || pvalid_host == nullptr || perf_host == nullptr)) || topk_host == nullptr)
+    return fail(MLT_EINVAL, "host buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  ScratchOwner& S = g_scr;
+  if (n > S.host_cap_n || g_F != S.host_cap_F || S.h_topk == nullptr) {
+    cudaDeviceSynchronize();
+    cudaFree(S.h_feats);
+    cudaFree(S.h_pvalid);
+    cudaFree(S.h_perf);
+    cudaFree(S.h_topk);
+    S.h_feats = nullptr;
+    S.h_pvalid = S.h_perf = nullptr;
+    S.h_topk = nullptr;
+    S.host_cap_n = -1;
+    const long long cap = n < 1024 ? 1024 : n;
+    if (cudaMalloc(&S.h_feats, sizeof(float) * cap * g_F) != cudaSuccess ||
+        cudaMalloc(&S.h_pvalid, sizeof(float) * cap) != cudaSuccess ||
+        cudaMalloc(&S.h_perf, sizeof(float) * cap) != cudaSuccess ||
+        cudaMalloc(&S.h_topk, sizeof(int64_t) * kMaxK) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(MLT_ENOMEM, "cannot allocate device staging for host buffers");
+    }
+    S.host_cap_n = cap;
+    S.host_cap_F = g_F;
+  }
+  if (n > 0)
+    MLT_CUDA(cudaMemcpyAsync(S.h_feats, feats_host, sizeof(float) * n * g_F, cudaMemcpyHostToDevice, st),
+             "feature upload");
+  rc = run_screen(st, S.h_feats, nullptr, n, thr, k, S.h_pvalid, S.h_perf, S.h_topk);
+  if (rc != MLT_OK) return rc;
+  if (n > 0) {
+    MLT_CUDA(cudaMemcpyAsync(pvalid_host, S.h_pvalid, sizeof(float) * n, cudaMemcpyDeviceToHost, st), "pvalid download");
+    MLT_CUDA(cudaMemcpyAsync(perf_host, S.h_perf, sizeof(float) * n, cudaMemcpyDeviceToHost, st), "perf download");
+  }
+  MLT_CUDA(cudaMemcpyAsync(topk_host, S.h_topk, sizeof(int64_t) * k, cudaMemcpyDeviceToHost, st), "top-k download");
+  MLT_CUDA(cudaStreamSynchronize(st), "stream synchronize");
+  return MLT_OK;
+}
+
+int mlt_decode_knobs(void* stream, const int32_t* radices, const float* option_values, int n_knobs,
+                     const mlt_feat_op* program, int F, int64_t first_index, int64_t n, uint8_t* out_knobs,
+                     float* out_feats) {
+  if (n < 0 || n > 0x7FFFFFFFLL) return fail(MLT_EINVAL, "n must lie in [0, 2^31-1]");
+  DecodeParams d;
+  int rc = build_decoder(radices, option_values, n_knobs, program, F, first_index, n, &d);
+  if (rc != MLT_OK) return rc;
+  if (n == 0) return MLT_OK;
+  MLT_CUDA(launch_decode_rows(d, n, out_knobs, out_feats, static_cast<cudaStream_t>(stream)), "decode launch");
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_launches += 1;
+  return MLT_OK;
+}
+
+int mlt_sync_status(void* stream) {
+  MLT_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream synchronize");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_scr.err == nullptr) return MLT_OK;
+  unsigned int word = 0;
+  MLT_CUDA(cudaMemcpy(&word, g_scr.err, sizeof(word), cudaMemcpyDeviceToHost), "error word read");
+  if (word == 0) return MLT_OK;
+  MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(word)), "error word reset");
+  if (word & kErrWaitTimeout) return fail(MLT_ETIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
+  return fail(MLT_ECUDA, "device-side bookkeeping error (error word 0x%x)", word);
+}
+
+int mlt_last_survivor_count(void* stream, int64_t* count_out) {
+  if (count_out == nullptr) return fail(MLT_EINVAL, "count_out must be non-NULL");
+  MLT_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream synchronize");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_scr.state == nullptr) {
+    *count_out = 0;
+    return MLT_OK;
+  }
+  unsigned int s = 0;
+  MLT_CUDA(cudaMemcpy(&s, &g_scr.state->survivors, sizeof(s), cudaMemcpyDeviceToHost), "survivor count read");
+  *count_out = s;
+  return MLT_OK;
+}
+
+int mlt_profile_phases(int enable) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_profile = enable != 0;
+  g_events_used = 0;
+  return MLT_OK;
+}
+
+int mlt_phase_times(float* out_ms, int n_phases, int64_t* n_calls_out) {
+  if (out_ms == nullptr || n_calls_out == nullptr || n_phases < 0)
+    return fail(MLT_EINVAL, "out_ms and n_calls_out must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  double sum[kPhases] = {0, 0, 0, 0};
+  const size_t calls = g_events_used / (kPhases + 1);
+  for (size_t c = 0; c < calls; ++c) {
+    cudaEvent_t* ev = &g_events[c * (kPhases + 1)];
+    MLT_CUDA(cudaEventSynchronize(ev[kPhases]), "cudaEventSynchronize");
+    for (int p = 0; p < kPhases; ++p) {
+      float ms = 0.0f;
+      MLT_CUDA(cudaEventElapsedTime(&ms, ev[p], ev[p + 1]), "cudaEventElapsedTime");
+      sum[p] += ms;
+    }
+  }
+  for (int p = 0; p < n_phases && p < kPhases; ++p) out_ms[p] = static_cast<float>(sum[p]);
+  *n_calls_out = static_cast<int64_t>(calls);
+  g_events_used = 0;
+  return MLT_OK;
+}
+
+int64_t mlt_kernel_launches(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  return g_launches;
+}
+
+const char* mlt_last_error(void) { return t_err.c_str(); }
+
+}  // extern "C"

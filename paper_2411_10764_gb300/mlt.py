@@ -1,0 +1,246 @@
+"""Python binding of libmlt (ctypes): argument marshalling only.
+
+Every step of screening runs in the CUDA library; this module only turns
+torch tensors / numpy arrays into pointers and sizes, passes the current
+CUDA stream, and raises MltError on a non-zero status.  There is no CPU
+fallback: if libmlt.so cannot be built or loaded, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import re
+import threading
+
+import numpy as np
+
+from . import _build
+
+MLT_MODEL_V, MLT_MODEL_P, MLT_MODEL_A = 0, 1, 2
+STATUS = {0: "MLT_OK", -1: "MLT_EINVAL", -2: "MLT_ENOMODEL", -3: "MLT_ECUDA", -4: "MLT_ENOMEM",
+          -5: "MLT_ETIMEOUT"}
+
+NODE_DTYPE = np.dtype(
+    [("feature", "<i4"), ("value", "<f4"), ("default_left", "u1"), ("pad", "u1", (3,))]
+)
+OP_DTYPE = np.dtype([("op", "<i4"), ("a", "<i4"), ("b", "<i4"), ("c", "<f4")])
+
+HEADER = os.path.join(_build.ROOT, "include", "mlt.h")
+
+
+class MltError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"{STATUS.get(code, code)}: {message}")
+        self.code = code
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def lib(build_if_missing: bool = True):
+    """Load libmlt.so (building it first when missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if build_if_missing:
+            _build.build()
+        if not os.path.exists(_build.LIB_PATH):
+            raise RuntimeError(f"libmlt.so missing at {_build.LIB_PATH}")
+        L = C.CDLL(_build.LIB_PATH)
+        P, i32, i64, f32 = C.c_void_p, C.c_int, C.c_int64, C.c_float
+        sig = {
+            "mlt_set_num_features": [i32],
+            "mlt_load_ensemble": [i32, P, i32, i32],
+            "mlt_free_ensemble": [i32],
+            "mlt_validity_cut": [f32, P],
+            "mlt_screen": [P, P, i64, f32, i32, P, P, P],
+            "mlt_screen_host": [P, P, i64, f32, i32, P, P, P],
+            "mlt_decode_knobs": [P, P, P, i32, P, i32, i64, i64, P, P],
+            "mlt_screen_decoded": [P, P, P, i32, P, i64, i64, f32, i32, P, P, P],
+            "mlt_sync_status": [P],
+            "mlt_last_survivor_count": [P, P],
+            "mlt_profile_phases": [i32],
+            "mlt_phase_times": [P, i32, P],
+        }
+        for name, args in sig.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = i32
+        L.mlt_kernel_launches.argtypes = []
+        L.mlt_kernel_launches.restype = i64
+        L.mlt_last_error.argtypes = []
+        L.mlt_last_error.restype = C.c_char_p
+        _lib = L
+        return L
+
+
+def declared_symbols() -> list[str]:
+    """Every function the C header declares."""
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(mlt_\w+)\s*\(", text, re.M)))
+
+
+def _check(rc: int):
+    if rc != 0:
+        msg = lib().mlt_last_error()
+        raise MltError(rc, msg.decode() if msg else "")
+
+
+def _stream_ptr(stream=None):
+    import torch
+
+    s = torch.cuda.current_stream() if stream is None else stream
+    return C.c_void_p(s.cuda_stream)
+
+
+def _dptr(t):
+    return C.c_void_p(0 if t is None else t.data_ptr())
+
+
+# ---------------------------------------------------------------------------
+# Model management
+# ---------------------------------------------------------------------------
+
+def set_num_features(F: int) -> None:
+    _check(lib().mlt_set_num_features(int(F)))
+
+
+def load_ensemble(model_id: int, nodes: np.ndarray, n_trees: int, depth: int) -> None:
+    nodes = np.ascontiguousarray(nodes)
+    if nodes.dtype.itemsize != 12:
+        raise ValueError("nodes must use the 12-byte slot layout")
+    if nodes.size != n_trees * ((2 << depth) - 1):
+        raise ValueError("node array size does not match n_trees and depth")
+    _check(lib().mlt_load_ensemble(int(model_id), nodes.ctypes.data, int(n_trees), int(depth)))
+
+
+def free_ensemble(model_id: int) -> None:
+    _check(lib().mlt_free_ensemble(int(model_id)))
+
+
+def validity_cut(thr: float) -> float:
+    out = C.c_float()
+    _check(lib().mlt_validity_cut(C.c_float(thr), C.byref(out)))
+    return out.value
+
+
+# ---------------------------------------------------------------------------
+# Screening
+# ---------------------------------------------------------------------------
+
+def _outputs(n, k, device, out_pvalid, out_perf, out_topk):
+    import torch
+
+    if out_pvalid is None:
+        out_pvalid = torch.empty(n, dtype=torch.float32, device=device)
+    if out_perf is None:
+        out_perf = torch.empty(n, dtype=torch.float32, device=device)
+    if out_topk is None:
+        out_topk = torch.empty(k, dtype=torch.int64, device=device)
+    return out_pvalid, out_perf, out_topk
+
+
+def screen(feats, thr: float, k: int, out_pvalid=None, out_perf=None, out_topk=None, stream=None):
+    """Screen a [n][F] fp32 CUDA tensor: returns (pvalid, perf, topk) tensors."""
+    import torch
+
+    if not (isinstance(feats, torch.Tensor) and feats.is_cuda and feats.dtype == torch.float32):
+        raise TypeError("feats must be a float32 CUDA tensor")
+    if not feats.is_contiguous() or feats.dim() != 2:
+        raise ValueError("feats must be a contiguous [n][F] tensor")
+    n = feats.shape[0]
+    pv, pf, tk = _outputs(n, k, feats.device, out_pvalid, out_perf, out_topk)
+    _check(lib().mlt_screen(_stream_ptr(stream), _dptr(feats), n, C.c_float(thr), int(k),
+                            _dptr(pv), _dptr(pf), _dptr(tk)))
+    return pv, pf, tk
+
+
+def screen_host(feats: np.ndarray, thr: float, k: int, out=None, stream=None):
+    """Screen a host [n][F] float32 array (copies in and out inside the call).
+
+    `out` may be a (pvalid, perf, topk) triple of host arrays (for example
+    pinned torch tensors' numpy views) to fill in place."""
+    feats = np.ascontiguousarray(feats, dtype=np.float32)
+    n = feats.shape[0]
+    if out is None:
+        out = (np.empty(n, np.float32), np.empty(n, np.float32), np.empty(k, np.int64))
+    pv, pf, tk = out
+    _check(lib().mlt_screen_host(_stream_ptr(stream), feats.ctypes.data, n, C.c_float(thr), int(k),
+                                 pv.ctypes.data, pf.ctypes.data, tk.ctypes.data))
+    return pv, pf, tk
+
+
+def _decoder_args(radices, option_values, program):
+    r = np.ascontiguousarray(radices, dtype=np.int32)
+    ov = np.ascontiguousarray(option_values, dtype=np.float32)
+    prog = np.ascontiguousarray(program)
+    if prog.dtype.itemsize != 16:
+        raise ValueError("program must use the 16-byte op layout")
+    return r, ov, prog
+
+
+def decode_knobs(radices, option_values, program, first_index: int, n: int, device="cuda",
+                 want_knobs=True, want_feats=True, stream=None):
+    """(knobs [n][K] uint8, feats [n][F] fp32) CUDA tensors (None if not wanted)."""
+    import torch
+
+    r, ov, prog = _decoder_args(radices, option_values, program)
+    knobs = torch.empty((n, r.size), dtype=torch.uint8, device=device) if want_knobs else None
+    feats = torch.empty((n, prog.size), dtype=torch.float32, device=device) if want_feats else None
+    _check(lib().mlt_decode_knobs(_stream_ptr(stream), r.ctypes.data, ov.ctypes.data, r.size,
+                                  prog.ctypes.data, prog.size, int(first_index), int(n),
+                                  _dptr(knobs), _dptr(feats)))
+    return knobs, feats
+
+
+def screen_decoded(radices, option_values, program, first_index: int, n: int, thr: float, k: int,
+                   device="cuda", out_pvalid=None, out_perf=None, out_topk=None, stream=None):
+    """Screen candidates first_index .. first_index+n-1 of a knob space."""
+    r, ov, prog = _decoder_args(radices, option_values, program)
+    pv, pf, tk = _outputs(n, k, device, out_pvalid, out_perf, out_topk)
+    _check(lib().mlt_screen_decoded(_stream_ptr(stream), r.ctypes.data, ov.ctypes.data, r.size,
+                                    prog.ctypes.data, int(first_index), int(n), C.c_float(thr),
+                                    int(k), _dptr(pv), _dptr(pf), _dptr(tk)))
+    return pv, pf, tk
+
+
+def sync_status(stream=None) -> None:
+    _check(lib().mlt_sync_status(_stream_ptr(stream)))
+
+
+def last_survivor_count(stream=None) -> int:
+    out = C.c_int64()
+    _check(lib().mlt_last_survivor_count(_stream_ptr(stream), C.byref(out)))
+    return int(out.value)
+
+
+PHASES = ("v_pass", "compaction", "p_pass", "topk")
+
+
+def profile_phases(enable: bool) -> None:
+    _check(lib().mlt_profile_phases(1 if enable else 0))
+
+
+def phase_times():
+    """({phase: summed ms}, recorded calls) since profiling was enabled."""
+    out = (C.c_float * 4)()
+    calls = C.c_int64()
+    _check(lib().mlt_phase_times(out, 4, C.byref(calls)))
+    return dict(zip(PHASES, [float(v) for v in out])), int(calls.value)
+
+
+def kernel_launches() -> int:
+    return int(lib().mlt_kernel_launches())
+
+
+def load_workload_models(w) -> None:
+    """Set F and load the workload's V and P ensembles."""
+    set_num_features(w.cfg.F if w.feats is None else w.feats.shape[1])
+    load_ensemble(MLT_MODEL_V, w.v.nodes, w.v.n_trees, w.v.depth)
+    load_ensemble(MLT_MODEL_P, w.p.nodes, w.p.n_trees, w.p.depth)

@@ -1,0 +1,191 @@
+"""GPU parity: the CUDA library against the oracle, element by element, on the
+same seeded inputs.  Decisions, survivor sets, top-k lists and P scores are
+bit-exact (fp32 leaf sums in tree order on both sides); pvalid is within
+1e-6 relative (device expf vs. host exp)."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2411_10764_gb300 import mlt
+from paper_2411_10764_gb300 import workloads as W
+from screening import (THREADS, assert_parity, assert_pvalid, assert_same_bits, gpu_screen,
+                       oracle_feats, oracle_screen, topk_from_scores)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    import torch
+
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    mlt.lib()
+
+
+# sizes that span several 256-candidate tiles and end on a ragged tile
+SMALL = {1: 4096, 2: 20000, 3: 9001, 4: 30000, 5: 5003}
+
+
+@pytest.mark.parametrize("cid", [1, 2, 3, 4, 5])
+def test_small_workloads_match_oracle(cid):
+    w = W.make_workload(cid, seed=1, n=SMALL[cid])
+    if w.decoder is not None:
+        w.first_index = 1234567
+    assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+@pytest.mark.parametrize("cid", [1, 3])
+def test_second_seed(cid):
+    w = W.make_workload(cid, seed=7, n=3000)
+    assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+def test_empty_batch():
+    w = W.make_workload(1, seed=1, n=0)
+    pv, pf, tk, s = gpu_screen(w)
+    assert pv.size == 0 and pf.size == 0 and s == 0
+    assert np.all(tk == -1)
+
+
+@pytest.mark.parametrize("n", [1, 31, 32, 33, 255, 257])
+def test_tiny_and_ragged_batches(n):
+    w = W.make_workload(1, seed=3, n=n)
+    assert_parity(gpu_screen(w, k=8), oracle_screen(w, k=8))
+
+
+@pytest.mark.parametrize("k", [1, 7, 2048, 16384])
+def test_k_sizes_including_more_than_survivors(k):
+    w = W.make_workload(2, seed=1, n=5000)
+    assert_parity(gpu_screen(w, k=k), oracle_screen(w, k=k))
+
+
+@pytest.mark.parametrize("thr", [1e-6, 0.999999, 0.3, 0.75])
+def test_thresholds_all_none_some(thr):
+    w = W.make_workload(1, seed=1, n=4096)
+    assert_parity(gpu_screen(w, thr=thr), oracle_screen(w, thr=thr))
+
+
+def test_missing_values_in_full_tables():
+    w = W.make_workload(1, seed=1, n=6000)
+    rng = np.random.default_rng(5)
+    x = w.feats.copy()
+    x[rng.random(size=x.shape) < 0.25] = np.nan
+    x[rng.random(size=x.shape) < 0.02] = np.inf
+    x[rng.random(size=x.shape) < 0.02] = -np.inf
+    x[:3] = np.nan  # rows entirely missing
+    assert_parity(gpu_screen(w, feats=x), oracle_screen(w, feats=x))
+
+
+def test_duplicate_rows_tie_break_by_index():
+    w = W.make_workload(2, seed=1, n=8000)
+    x = w.feats.copy()
+    x[1::2] = x[0::2]  # every score appears twice
+    x[5000:] = x[17]  # a large block of identical candidates
+    g = gpu_screen(w, feats=x, k=512)
+    o = oracle_screen(w, feats=x, k=512)
+    assert_parity(g, o)
+
+
+def test_unbalanced_shallow_trees_use_padded_full_tables():
+    cfg = W.ScreenConfig(98, "unbalanced-d7", 7000, 40, 60, 7, 90, 7, 0.5, 100, None,
+                         shape="unbalanced", split_dist="zipf", nan_frac=0.2, dup_frac=0.05)
+    x = W.make_features(W.CONFIGS[5], 2, 7000)[:, :40].copy()
+    th = W._QuantileThresholds(x[:4096])
+    w = W.Workload(cfg, 7000, x, None, 0, W.make_ensemble(cfg, "V", th, 4),
+                   W.make_ensemble(cfg, "P", th, 4), 0.5, 100)
+    assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+@pytest.mark.parametrize("F", [30, 7])
+def test_feature_counts_not_multiple_of_four(F):
+    cfg = W.ScreenConfig(97, f"f{F}", 3000, F, 40, 6, 50, 5, 0.5, 64, None)
+    x = W.make_features(W.CONFIGS[1], 3, 3000)
+    x = np.ascontiguousarray(np.tile(x, (1, 2))[:, :F])
+    th = W._QuantileThresholds(x[:2048])
+    w = W.Workload(cfg, 3000, x, None, 0, W.make_ensemble(cfg, "V", th, 5),
+                   W.make_ensemble(cfg, "P", th, 5), 0.5, 64)
+    assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+def test_unaligned_feature_pointer():
+    import torch
+
+    w = W.make_workload(1, seed=1, n=2000)
+    mlt.load_workload_models(w)
+    buf = torch.empty(w.feats.size + 1, dtype=torch.float32, device="cuda")
+    x = buf[1:].view(w.feats.shape)  # 4-byte aligned only
+    x.copy_(torch.from_numpy(w.feats))
+    pv, pf, tk = mlt.screen(x, w.thr, w.k)
+    mlt.sync_status()
+    g = (pv.cpu().numpy(), pf.cpu().numpy(), tk.cpu().numpy(), mlt.last_survivor_count())
+    assert_parity(g, oracle_screen(w))
+
+
+def test_host_buffer_entry_point_matches_device_call():
+    w = W.make_workload(2, seed=2, n=12345)
+    g = gpu_screen(w)
+    pv, pf, tk = mlt.screen_host(w.feats, w.thr, w.k)
+    assert_same_bits(pv, g[0], "pvalid (host entry)")
+    assert_same_bits(pf, g[1], "perf (host entry)")
+    assert np.array_equal(tk, g[2])
+
+
+def test_decoded_knobs_and_features_bit_exact():
+    d = W.conv2d_decoder(seed=1)
+    for first, n in [(0, 4096), (16777216 - 5000, 5000), (987654, 3333)]:
+        knobs, feats = mlt.decode_knobs(d.radices, d.option_values, d.program, first, n)
+        ok, of = O.features(d.radices, d.option_values, d.program, first, n, threads=THREADS)
+        assert np.array_equal(knobs.cpu().numpy(), ok)
+        assert_same_bits(feats.cpu().numpy(), of, "decoded features")
+
+
+def test_decoded_screen_equals_materialised_screen():
+    w = W.make_workload(4, seed=1, n=20000)
+    w.first_index = 5_000_000
+    d = w.decoder
+    g_dec = gpu_screen(w)
+    _, feats = mlt.decode_knobs(d.radices, d.option_values, d.program, w.first_index, w.n)
+    import torch
+
+    pv, pf, tk = mlt.screen(feats, w.thr, w.k)
+    assert_same_bits(pf.cpu().numpy(), g_dec[1], "perf decoded vs materialised")
+    assert np.array_equal(tk.cpu().numpy() + w.first_index, g_dec[2])
+    torch.cuda.synchronize()
+
+
+def test_full_size_config2_all_outputs():
+    w = W.make_workload(2, seed=1)
+    assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+def _sampled_full_size(cid, n_sample=1500):
+    w = W.make_workload(cid, seed=1)
+    gpv, gpf, gtk, gs = gpu_screen(w)
+    # selection logic: exact at full size against a sort of the scores
+    want, s = topk_from_scores(gpf, w.k, w.first_index)
+    assert s == gs
+    assert np.array_equal(gtk, want)
+    # scores and decisions: sampled rows, the kept rows and the rows nearest
+    # to the validity cut and to the k-th score
+    rng = np.random.default_rng(11)
+    tau = O.tau(w.thr)
+    sig_tau = O.sigmoid(tau)
+    near_cut = np.argsort(np.abs(gpv.astype(np.float64) - sig_tau))[:200]
+    kept = gtk[gtk >= 0] - w.first_index
+    finite = gpf > -np.inf
+    kth = gpf[kept[-1]] if kept.size else 0.0
+    near_k = np.nonzero(finite)[0][np.argsort(np.abs(gpf[finite] - kth))[:200]]
+    rows = np.unique(np.concatenate([rng.choice(w.n, n_sample, replace=False), kept, near_cut,
+                                     near_k]))
+    x = oracle_feats(w, rows)
+    opv, opf, ovalid, _ = O.screen_rows(x, w.v, w.p, w.thr, threads=THREADS)
+    assert_same_bits(gpf[rows], opf, "perf (sampled)")
+    assert_pvalid(gpv[rows], opv)
+    n_near = int(np.sum(np.abs(gpf[finite] - kth) <= 1e-6 * abs(kth)))
+    print(f"config {cid}: survivors {gs}/{w.n}, {rows.size} rows checked, "
+          f"{n_near} scores within 1e-6 of the k-th")
+
+
+@pytest.mark.parametrize("cid", [3, 4, 5])
+def test_full_size_sampled(cid):
+    _sampled_full_size(cid)
