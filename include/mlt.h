@@ -194,6 +194,13 @@ int mlt_profile_phases(int enable);
  * *n_calls_out receives the number of recorded calls.  Clears the records. */
 int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
 
+/* Tuning: fix the launch shape of the walk over model `model_id`'s trees:
+ * candidates per CTA (threads: 32, 64, 128 or 256), trees per shared-memory
+ * chunk (1, 2, 4, 8 or 16) and chunk buffers (2 or 3); 0 = let the library
+ * choose (the default).  A shape that does not fit shared memory falls back
+ * to the library's choice.  Results do not depend on the shape.  Host-only. */
+int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf);
+
 /* Cumulative number of GPU kernels this library has launched. */
 int64_t mlt_kernel_launches(void);
 

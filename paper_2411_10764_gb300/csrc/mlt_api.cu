@@ -60,7 +60,6 @@ struct ScratchOwner {
   Scratch s;
   void* block = nullptr;  // one allocation for everything sized by n
   SelectState* state = nullptr;
-  unsigned long long* sel = nullptr;
   unsigned int* err = nullptr;
   // host-buffer entry point staging
   long long host_cap_n = -1;
@@ -83,6 +82,8 @@ size_t g_events_used = 0;
 Model g_models[3];
 ScratchOwner g_scr;
 int g_optin = -1;
+int g_sms = -1;
+ShapeOverride g_shape[3];
 
 size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
 
@@ -101,6 +102,17 @@ int smem_optin() {
     g_optin = v;
   }
   return g_optin;
+}
+
+int sm_count() {
+  if (g_sms < 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return 1;
+    g_sms = v;
+  }
+  return g_sms;
 }
 
 void free_model(Model& m) {
@@ -123,7 +135,6 @@ int ensure_scratch(long long n) {
     MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(unsigned int)), "cudaMemset(error word)");
     MLT_CUDA(cudaMalloc(&g_scr.state, sizeof(SelectState)), "cudaMalloc(select state)");
     MLT_CUDA(cudaMemset(g_scr.state, 0, sizeof(SelectState)), "cudaMemset(select state)");
-    MLT_CUDA(cudaMalloc(&g_scr.sel, sizeof(unsigned long long) * kMaxK), "cudaMalloc(selection)");
     g_scr.device = dev;
   }
   if (n > g_scr.cap_n) {
@@ -133,7 +144,7 @@ int ensure_scratch(long long n) {
     const size_t b_tiles = align16(words * 4);  // tiles are >= 32 candidates
     const size_t b_rows = align16(cap * 4);
     const size_t b_keys = align16(cap * 8);
-    const size_t total = b_masks + 2 * b_tiles + b_rows + b_keys;
+    const size_t total = b_masks + 2 * b_tiles + b_rows + 2 * b_keys;
     if (g_scr.block != nullptr) {
       cudaDeviceSynchronize();
       cudaFree(g_scr.block);
@@ -156,11 +167,12 @@ int ensure_scratch(long long n) {
     g_scr.s.rows = reinterpret_cast<uint32_t*>(p);
     p += b_rows;
     g_scr.s.keys = reinterpret_cast<unsigned long long*>(p);
+    p += b_keys;
+    g_scr.s.cand = reinterpret_cast<unsigned long long*>(p);
     g_scr.block = blk;
     g_scr.cap_n = cap;
   }
   g_scr.s.state = g_scr.state;
-  g_scr.s.sel = g_scr.sel;
   g_scr.s.err = g_scr.err;
   return MLT_OK;
 }
@@ -203,9 +215,12 @@ int check_models(int dev) {
   return MLT_OK;
 }
 
-ScreenShape plan_for(const DeviceModel& dm, int F) {
-  if (dm.kind == kTableFull) return plan_full(F, dm.depth, dm.n_trees, dm.tree_bytes, smem_optin());
-  return plan_compact(F, smem_optin());
+ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov) {
+  ScreenShape s = dm.kind == kTableFull
+                      ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
+                      : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
+  if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf)) return plan_for(dm, F, n_eff, ShapeOverride());
+  return s;
 }
 
 int build_decoder(const int32_t* radices, const float* option_values, int n_knobs,
@@ -281,12 +296,15 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
   dm.n_trees = n_trees;
   dm.depth = depth;
   if (depth <= kMaxFullDepth) {
-    const uint32_t I = (1u << depth) - 1u, L = 1u << depth;
-    const size_t tb = align16(static_cast<size_t>(I) * 8 + static_cast<size_t>(L) * 4);
+    const FullLayout lay = full_layout(depth);
+    const size_t tb = lay.bytes;
     dm.kind = kTableFull;
-    dm.tree_bytes = static_cast<uint32_t>(tb);
+    dm.tree_bytes = lay.bytes;
     out.assign(tb * n_trees, 0);
+    const int inner = (1 << depth) - 1;  // internal heap slots of the complete tree
     std::vector<float> inherit(slots);
+    std::vector<float> thr_of(inner);
+    std::vector<uint32_t> meta_of(inner);
     for (int t = 0; t < n_trees; ++t) {
       const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
       unsigned char* dst = out.data() + tb * t;
@@ -305,18 +323,25 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
           inherit[j] = inherit[(j - 1) / 2];  // below a leaf: copy it down
         else
           inherit[j] = 0.0f;
-        if (static_cast<uint32_t>(j) < I) {
-          float thr = 0.0f;
-          uint32_t meta = 0;
-          if (split) {
-            thr = nd.value;
-            meta = static_cast<uint32_t>(nd.feature) | (nd.default_left ? kMetaDefaultLeft : 0u);
-          }
-          std::memcpy(dst + 8 * j, &thr, 4);
-          std::memcpy(dst + 8 * j + 4, &meta, 4);
+        if (j < inner) {
+          thr_of[j] = split ? nd.value : 0.0f;
+          meta_of[j] = split ? (static_cast<uint32_t>(nd.feature) | (nd.default_left ? kMetaDefaultLeft : 0u)) : 0u;
+        }
+      }
+      for (uint32_t j = 0; j < static_cast<uint32_t>(inner); ++j) {
+        if (j < lay.n_top) {
+          std::memcpy(dst + 8 * j, &thr_of[j], 4);
+          std::memcpy(dst + 8 * j + 4, &meta_of[j], 4);
+        } else if (j < lay.n_inner) {
+          std::memcpy(dst + lay.off_thr + 4 * (j - lay.n_top), &thr_of[j], 4);
+          std::memcpy(dst + lay.off_meta + 4 * (j - lay.n_top), &meta_of[j], 4);
         } else {
-          const float leaf = inherit[j];
-          std::memcpy(dst + 8 * I + 4 * (j - I), &leaf, 4);
+          unsigned char* rec = dst + lay.off_last + 16 * (j - lay.n_inner);
+          const float left = inherit[2 * j + 1], right = inherit[2 * j + 2];
+          std::memcpy(rec, &thr_of[j], 4);
+          std::memcpy(rec + 4, &meta_of[j], 4);
+          std::memcpy(rec + 8, &left, 4);
+          std::memcpy(rec + 12, &right, 4);
         }
       }
     }
@@ -369,7 +394,9 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   if (rc != MLT_OK) return rc;
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
-  const ScreenShape sv = plan_for(V, g_F), sp = plan_for(P, g_F);
+  // the P pass walks the survivors; plan it for about half the batch
+  const ScreenShape sv = plan_for(V, g_F, n, g_shape[MLT_MODEL_V]);
+  const ScreenShape sp = plan_for(P, g_F, (n + 1) / 2, g_shape[MLT_MODEL_P]);
   if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
   const Scratch& s = g_scr.s;
   TraverseArgs a{};
@@ -385,6 +412,7 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   a.masks = s.masks;
   a.tile_counts = s.tile_counts;
   a.keys = s.keys;
+  a.hist = s.state->hist;
   a.err = s.err;
   a.decode = dec != nullptr;
 
@@ -410,9 +438,10 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
     MLT_CUDA(cudaEventRecord(ev[0], st), "cudaEventRecord");
   }
   const long long tiles_v = (n + sv.threads - 1) / sv.threads;
-  MLT_CUDA(launch_traverse(V, av, dec, sv, tiles_v, st), "V pass launch");
+  MLT_CUDA(dec ? launch_traverse_dec(V, av, *dec, sv, tiles_v, st) : launch_traverse(V, av, sv, tiles_v, st),
+           "V pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[1], st), "cudaEventRecord");
-  MLT_CUDA(launch_compact(s, n, sv.threads, tiles_v, k, st), "compaction launch");
+  MLT_CUDA(launch_compact(s, n, sv.threads, tiles_v, st), "compaction launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[2], st), "cudaEventRecord");
 
   TraverseArgs ap = a;
@@ -424,11 +453,12 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   ap.nbuf = sp.nbuf;
   ap.max_depth = P.depth;
   const long long tiles_p = (n + sp.threads - 1) / sp.threads;
-  MLT_CUDA(launch_traverse(P, ap, dec, sp, tiles_p, st), "P pass launch");
+  MLT_CUDA(dec ? launch_traverse_dec(P, ap, *dec, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
+           "P pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[3], st), "cudaEventRecord");
-  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, st), "top-k launch");
+  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, sm_count(), st), "top-k launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
-  g_launches += (tiles_v > 0 ? 1 : 0) + 1 + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + kRadixPasses + 2;
+  g_launches += (tiles_v > 0 ? 1 : 0) + 1 + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
   return MLT_OK;
 }
 
@@ -632,6 +662,21 @@ int mlt_phase_times(float* out_ms, int n_phases, int64_t* n_calls_out) {
   for (int p = 0; p < n_phases && p < kPhases; ++p) out_ms[p] = static_cast<float>(sum[p]);
   *n_calls_out = static_cast<int64_t>(calls);
   g_events_used = 0;
+  return MLT_OK;
+}
+
+int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf) {
+  if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
+  if (!(threads == 0 || threads == 32 || threads == 64 || threads == 128 || threads == 256))
+    return fail(MLT_EINVAL, "threads must be 0, 32, 64, 128 or 256");
+  if (!(chunk_trees == 0 || chunk_trees == 1 || chunk_trees == 2 || chunk_trees == 4 || chunk_trees == 8 ||
+        chunk_trees == 16))
+    return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8 or 16");
+  if (!(nbuf == 0 || nbuf == 2 || nbuf == 3)) return fail(MLT_EINVAL, "nbuf must be 0, 2 or 3");
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_shape[model_id].threads = threads;
+  g_shape[model_id].chunk_trees = chunk_trees;
+  g_shape[model_id].nbuf = nbuf;
   return MLT_OK;
 }
 

@@ -27,12 +27,19 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 // Packed device tables
 // ---------------------------------------------------------------------------
 // Full table (depth D <= kMaxFullDepth): every tree is stored as a complete
-// binary tree of depth D, `tree_bytes` apart (a multiple of 16):
-//   I = 2^D - 1 internal records {float threshold; uint32 meta}, heap order,
-//     meta bits 0..30 = feature index, bit 31 = NaN goes left;
-//   L = 2^D leaf values (float), heap order of the last level.
+// binary tree of depth D, `tree_bytes` apart (a multiple of 16).  A node has
+// a threshold (float) and a meta word (bits 0..30 feature index, bit 31 NaN
+// goes left); its heap index is j (children 2j+1, 2j+2).  Each level is laid
+// out for the way a warp reads it (FullLayout below):
+//   levels [0, top)      : 8-byte records {threshold, meta} -- few distinct
+//                          nodes, mostly broadcast reads;
+//   levels [top, D-1)    : thresholds and metas in two 4-byte arrays -- a
+//                          32-lane gather of 4-byte words;
+//   level D-1 (last)     : 16-byte records {threshold, meta, left leaf,
+//                          right leaf} -- the last split and both leaves in
+//                          one load.
 // A shallower leaf is replicated into every leaf slot below it (its
-// pass-through internal records test feature 0; any path gives the leaf).
+// pass-through nodes test feature 0; any path gives the leaf).
 //
 // Compact table (any depth <= kMaxDepth): uint32 offsets[n_trees] (in
 // records, from the start of the record area, which begins at byte
@@ -42,6 +49,27 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 //   bits 16..29 = index of the left child within the tree (right = left+1),
 //   bits 0..15 = feature index.
 enum TableKind : int { kTableFull = 0, kTableCompact = 1 };
+
+struct FullLayout {
+  uint32_t top;        // levels held as 8-byte records
+  uint32_t n_top;      // nodes in levels [0, top)
+  uint32_t n_inner;    // nodes in levels [0, D-1)
+  uint32_t off_thr;    // byte offset of the middle-level thresholds
+  uint32_t off_meta;   // byte offset of the middle-level metas
+  uint32_t off_last;   // byte offset of the last-level 16-byte records
+  uint32_t bytes;      // bytes per tree (multiple of 16)
+};
+
+__host__ __device__ constexpr FullLayout full_layout(int D) {
+  const uint32_t top = D - 1 < 4 ? static_cast<uint32_t>(D - 1) : 4u;
+  const uint32_t n_top = (1u << top) - 1u;
+  const uint32_t n_inner = (1u << (D - 1)) - 1u;
+  const uint32_t off_thr = n_top * 8u;
+  const uint32_t off_meta = off_thr + (n_inner - n_top) * 4u;
+  const uint32_t off_last = (off_meta + (n_inner - n_top) * 4u + 15u) & ~15u;
+  const uint32_t bytes = off_last + (1u << (D - 1)) * 16u;
+  return FullLayout{top, n_top, n_inner, off_thr, off_meta, off_last, bytes};
+}
 
 constexpr uint32_t kMetaLeaf = 1u << 30;
 constexpr uint32_t kMetaDefaultLeft = 1u << 31;
@@ -74,19 +102,21 @@ struct DecodeParams {
 // ---------------------------------------------------------------------------
 // Scratch and top-k selection state
 // ---------------------------------------------------------------------------
-constexpr int kRadixBins = 2048;  // 11-bit digits
-constexpr int kRadixPasses = 6;   // 11+11+11+11+11+9 = 64 bits
+// The P pass histograms the top kTopBits bits of every rank key; the top-k
+// kernel reads it to find the bucket holding the k-th key, collects the keys
+// of that bucket and above (normally a few thousand), and sorts them in one
+// CTA.  kCollectCap is the most keys that sort in shared memory; a larger
+// collection (heavy ties) is narrowed by a radix select first.
+constexpr int kTopBits = 12;
+constexpr int kTopBins = 1 << kTopBits;
+constexpr int kCollectCap = 16384;
 
 struct SelectState {
-  unsigned long long prefix;  // key bits fixed so far
-  unsigned long long mask;    // which bits `prefix` fixes
-  unsigned int remaining;     // rank still to find among prefix-matching keys
-  unsigned int done;          // selection already determined
-  unsigned int ticket;        // blocks finished in the current pass
-  unsigned int n_sel;         // keys gathered
-  unsigned int survivors;     // valid candidates of the current batch
-  unsigned int k;             // requested k
-  unsigned int hist[kRadixBins];
+  unsigned int survivors;  // valid candidates of the current batch
+  unsigned int n_cand;     // keys collected for the final sort
+  unsigned int ticket;     // CTAs of the top-k kernel that finished
+  unsigned int pad;
+  unsigned int hist[kTopBins];
 };
 
 struct Scratch {
@@ -95,7 +125,7 @@ struct Scratch {
   uint32_t* tile_offsets = nullptr;  // [n_tiles] exclusive prefix
   uint32_t* rows = nullptr;          // [n] survivor positions, ascending
   unsigned long long* keys = nullptr;  // [n] (score, position) keys
-  unsigned long long* sel = nullptr;   // [kMaxK] selected keys
+  unsigned long long* cand = nullptr;  // [n] collected keys
   SelectState* state = nullptr;
   unsigned int* err = nullptr;       // device error word
 };
@@ -126,6 +156,7 @@ struct TraverseArgs {
   uint32_t* masks;
   uint32_t* tile_counts;
   unsigned long long* keys;
+  unsigned int* hist;      // P pass: key histogram (kTopBins)
   unsigned int* err;
   int decode;              // features built from candidate indices
 };
@@ -138,18 +169,32 @@ struct ScreenShape {
   int group;           // trees walked together per thread (ILP)
 };
 
+// Launch-shape override (mlt_tune_shape): 0 fields mean "choose".
+struct ShapeOverride {
+  int threads = 0;
+  int chunk_trees = 0;
+  int nbuf = 0;
+};
+
 // traverse.cu
-ScreenShape plan_full(int F, int depth, int n_trees, uint32_t tree_bytes, int device_smem_optin);
-ScreenShape plan_compact(int F, int device_smem_optin);
-cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, const DecodeParams* dec,
+// n_eff: candidates the pass is expected to walk (used for load balance).
+ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, int sms,
+                      int device_smem_optin, const ShapeOverride& ov);
+ScreenShape plan_compact(int F, long long n_eff, int sms, int device_smem_optin,
+                         const ShapeOverride& ov);
+cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args,
                             const ScreenShape& shape, long long n_tiles, cudaStream_t st);
+// traverse_dec.cu
+cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args,
+                                const DecodeParams& dec, const ScreenShape& shape,
+                                long long n_tiles, cudaStream_t st);
 cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* out_knobs,
                                float* out_feats, cudaStream_t st);
 
 // select.cu
-cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, int k,
+cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles,
                            cudaStream_t st);
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base,
-                        int64_t* out_topk, cudaStream_t st);
+                        int64_t* out_topk, int sms, cudaStream_t st);
 
 }  // namespace mlt

@@ -8,22 +8,24 @@
 // into the ascending list of survivor positions (stable, no atomics on the
 // order).  The P pass leaves one 64-bit key per survivor (score mapped to an
 // order-preserving integer, then ~position), so keys are unique and "k
-// largest keys" is exactly "k best by (score desc, position asc)".  A
-// most-significant-digit radix select (six passes of 11/11/11/11/11/9 bits)
-// finds the k-th key without any inter-CTA waiting: the last CTA of each
-// pass (ticket counter) picks the digit.  The <= k selected keys are then
-// sorted in one CTA (bitonic) and written as indices.
+// largest keys" is exactly "k best by (score desc, position asc)"; it also
+// counts the keys' top 12 bits in a histogram.  One top-k kernel then finds
+// the histogram bucket holding the k-th key, collects every key in that
+// bucket or above (a few thousand for the workloads here), and the last CTA
+// to finish (ticket counter, no waiting) sorts them in shared memory.  If
+// ties crowd more keys into the collection than shared memory holds, that
+// CTA first narrows them with an exact most-significant-digit radix select.
 #include "mlt_internal.cuh"
 
 namespace mlt {
 namespace {
 
 constexpr int kScanThreads = 1024;
-constexpr int kPassThreads = 256;
-constexpr int kSortThreads = 1024;
+constexpr int kTopkThreads = 512;
+constexpr int kSortMin = 8192;  // sort buffer entries (at least pow2(k))
 
 __global__ void __launch_bounds__(kScanThreads)
-    k_scan(const uint32_t* counts, uint32_t* offsets, long long n_tiles, SelectState* st, int k) {
+    k_scan(const uint32_t* counts, uint32_t* offsets, long long n_tiles, SelectState* st) {
   __shared__ unsigned part[kScanThreads];
   const int T = blockDim.x, tid = threadIdx.x;
   const long long per = (n_tiles + T - 1) / T;
@@ -45,17 +47,11 @@ __global__ void __launch_bounds__(kScanThreads)
     run += counts[i];
   }
   if (tid == T - 1) {
-    const unsigned total = part[T - 1];
-    st->survivors = total;
-    st->k = static_cast<unsigned>(k);
-    st->prefix = 0ull;
-    st->mask = 0ull;
-    st->remaining = total < static_cast<unsigned>(k) ? total : static_cast<unsigned>(k);
-    st->done = total <= static_cast<unsigned>(k) ? 1u : 0u;
+    st->survivors = part[T - 1];
+    st->n_cand = 0u;
     st->ticket = 0u;
-    st->n_sel = 0u;
   }
-  for (int i = tid; i < kRadixBins; i += T) st->hist[i] = 0u;
+  for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
 }
 
 __global__ void __launch_bounds__(256)
@@ -72,101 +68,9 @@ __global__ void __launch_bounds__(256)
   if ((m >> lane) & 1u) rows[base + __popc(m & ((1u << lane) - 1u))] = static_cast<uint32_t>(first + lane);
 }
 
-__device__ __forceinline__ int pass_shift(int pass) { return pass < 5 ? 53 - 11 * pass : 0; }
-__device__ __forceinline__ int pass_width(int pass) { return pass < 5 ? 11 : 9; }
-
-__global__ void __launch_bounds__(kPassThreads)
-    k_radix_pass(const unsigned long long* keys, SelectState* st, int pass) {
-  __shared__ unsigned hist[kRadixBins];
-  __shared__ unsigned part[kPassThreads];
-  __shared__ unsigned is_last;
-  if (st->done) return;  // written by an earlier kernel; uniform
+// Bitonic sort of sk[0, n2) in descending order (n2 a power of two).
+__device__ void sort_desc(unsigned long long* sk, int n2) {
   const int tid = threadIdx.x, T = blockDim.x;
-  const unsigned S = st->survivors;
-  const int shift = pass_shift(pass), width = pass_width(pass);
-  const int nb = 1 << width;
-  const unsigned long long dmask = (1ull << width) - 1ull;
-  const unsigned long long mask = st->mask, prefix = st->prefix;
-  const unsigned rem = st->remaining;  // read before the last CTA rewrites it
-  for (int i = tid; i < nb; i += T) hist[i] = 0u;
-  __syncthreads();
-  for (long long i = static_cast<long long>(blockIdx.x) * T + tid; i < S;
-       i += static_cast<long long>(gridDim.x) * T) {
-    const unsigned long long key = keys[i];
-    if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1u);
-  }
-  __syncthreads();
-  for (int i = tid; i < nb; i += T)
-    if (hist[i]) atomicAdd(&st->hist[i], hist[i]);
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) is_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
-  // Last CTA: pick the digit of the rem-th largest prefix-matching key.
-  // Thread t owns reversed positions [t*per, (t+1)*per): digits nb-1-r.
-  const int per = nb / T;  // nb is a multiple of T
-  unsigned local = 0;
-  for (int q = 0; q < per; ++q) {
-    const int d = nb - 1 - (tid * per + q);
-    const unsigned h = __ldcg(&st->hist[d]);
-    hist[d] = h;
-    local += h;
-  }
-  part[tid] = local;
-  __syncthreads();
-  for (int off = 1; off < T; off <<= 1) {
-    const unsigned v = tid >= off ? part[tid - off] : 0u;
-    __syncthreads();
-    part[tid] += v;
-    __syncthreads();
-  }
-  unsigned above = part[tid] - local;  // keys on digits above this thread's range
-  for (int q = 0; q < per; ++q) {
-    const int d = nb - 1 - (tid * per + q);
-    const unsigned h = hist[d];
-    if (above < rem && rem <= above + h) {
-      const unsigned left = rem - above;
-      st->remaining = left;
-      st->prefix = prefix | (static_cast<unsigned long long>(d) << shift);
-      st->mask = mask | (dmask << shift);
-      st->done = (left == h || pass == kRadixPasses - 1) ? 1u : 0u;
-    }
-    above += h;
-  }
-  __syncthreads();
-  for (int i = tid; i < kRadixBins; i += T) st->hist[i] = 0u;
-  if (tid == 0) st->ticket = 0u;
-}
-
-__global__ void __launch_bounds__(256)
-    k_gather(const unsigned long long* keys, SelectState* st, unsigned long long* sel, unsigned* err) {
-  const unsigned S = st->survivors;
-  const unsigned long long mask = st->mask, prefix = st->prefix;
-  const unsigned k = st->k;
-  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < S;
-       i += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const unsigned long long key = keys[i];
-    if ((key & mask) >= prefix) {
-      const unsigned p = atomicAdd(&st->n_sel, 1u);
-      if (p < k)
-        sel[p] = key;
-      else
-        atomicOr(err, kErrSelect);
-    }
-  }
-}
-
-__global__ void __launch_bounds__(kSortThreads)
-    k_sort_out(const SelectState* st, const unsigned long long* sel, int k, int n2, long long base,
-               int64_t* out) {
-  extern __shared__ __align__(16) unsigned long long sk[];
-  const int tid = threadIdx.x, T = blockDim.x;
-  const unsigned cnt_raw = st->n_sel;
-  const int cnt = static_cast<int>(cnt_raw < static_cast<unsigned>(k) ? cnt_raw : static_cast<unsigned>(k));
-  for (int i = tid; i < n2; i += T) sk[i] = i < cnt ? sel[i] : 0ull;
-  __syncthreads();
   for (int size = 2; size <= n2; size <<= 1) {
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
       for (int i = tid; i < (n2 >> 1); i += T) {
@@ -182,8 +86,132 @@ __global__ void __launch_bounds__(kSortThreads)
       __syncthreads();
     }
   }
+}
+
+__global__ void __launch_bounds__(kTopkThreads)
+    k_topk(const unsigned long long* keys, unsigned long long* cand, SelectState* st, int k, int cap,
+           long long base, int64_t* out, unsigned* err) {
+  extern __shared__ __align__(16) unsigned long long sk[];  // cap entries
+  __shared__ unsigned part[kTopkThreads];
+  __shared__ unsigned s_bin, s_last, s_digit, s_rem, s_h, s_cnt;
+  __shared__ unsigned h256[256];
+  const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31;
+  const unsigned S = st->survivors;
+  const unsigned kk = S < static_cast<unsigned>(k) ? S : static_cast<unsigned>(k);
+
+  // 1. bucket of the kk-th largest key: thread t owns the top bins
+  //    [nb-1-t*per, nb-1-(t+1)*per+1], scanned from the top
+  constexpr int per = kTopBins / kTopkThreads;
+  unsigned local = 0;
+  for (int q = 0; q < per; ++q) local += st->hist[kTopBins - 1 - (tid * per + q)];
+  part[tid] = local;
+  if (tid == 0) s_bin = kTopBins;  // nothing to select unless found
+  __syncthreads();
+  for (int off = 1; off < T; off <<= 1) {
+    const unsigned v = tid >= off ? part[tid - off] : 0u;
+    __syncthreads();
+    part[tid] += v;
+    __syncthreads();
+  }
+  unsigned above = part[tid] - local;
+  for (int q = 0; q < per; ++q) {
+    const int b = kTopBins - 1 - (tid * per + q);
+    const unsigned h = st->hist[b];
+    if (kk > 0 && above < kk && kk <= above + h) s_bin = static_cast<unsigned>(b);
+    above += h;
+  }
+  __syncthreads();
+  const unsigned long long bin = s_bin;
+
+  // 2. collect every key in that bucket or above (warp-aggregated appends)
+  for (long long i0 = static_cast<long long>(blockIdx.x) * T; i0 < S; i0 += static_cast<long long>(gridDim.x) * T) {
+    const long long i = i0 + tid;
+    unsigned long long key = 0;
+    bool take = false;
+    if (i < S) {
+      key = keys[i];
+      take = (key >> (64 - kTopBits)) >= bin;
+    }
+    const unsigned ball = __ballot_sync(0xFFFFFFFFu, take);
+    if (ball) {
+      const int leader = __ffs(ball) - 1;
+      unsigned pos0 = 0;
+      if (lane == leader) pos0 = atomicAdd(&st->n_cand, static_cast<unsigned>(__popc(ball)));
+      pos0 = __shfl_sync(0xFFFFFFFFu, pos0, leader);
+      if (take) cand[pos0 + __popc(ball & ((1u << lane) - 1u))] = key;
+    }
+  }
+
+  // 3. the last CTA to finish selects and sorts
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const unsigned m = *reinterpret_cast<volatile unsigned*>(&st->n_cand);
+  int n2 = 1;
+  while (n2 < static_cast<int>(kk)) n2 <<= 1;
+  if (m <= static_cast<unsigned>(cap)) {
+    // every collected key fits: sort them all, keep the first kk
+    int m2 = 1;
+    while (m2 < static_cast<int>(m)) m2 <<= 1;
+    for (int i = tid; i < m2; i += T) sk[i] = i < static_cast<int>(m) ? __ldcg(cand + i) : 0ull;
+    __syncthreads();
+    sort_desc(sk, m2);
+  } else {
+    // heavy ties: exact radix select of the kk-th key among the collected
+    // keys (8-bit digits from the top), then gather the kk keys above it
+    unsigned long long prefix = 0, mask = 0;
+    unsigned rem = kk;
+    for (int shift = 56; shift >= 0; shift -= 8) {
+      for (int i = tid; i < 256; i += T) h256[i] = 0u;
+      __syncthreads();
+      for (unsigned i = tid; i < m; i += T) {
+        const unsigned long long key = __ldcg(cand + i);
+        if ((key & mask) == prefix) atomicAdd(&h256[(key >> shift) & 0xFFull], 1u);
+      }
+      __syncthreads();
+      if (tid == 0) {
+        unsigned cum = 0;
+        for (int d = 255; d >= 0; --d) {
+          const unsigned h = h256[d];
+          if (cum + h >= rem) {
+            s_digit = static_cast<unsigned>(d);
+            s_rem = rem - cum;
+            s_h = h;
+            break;
+          }
+          cum += h;
+        }
+      }
+      __syncthreads();
+      prefix |= static_cast<unsigned long long>(s_digit) << shift;
+      mask |= 0xFFull << shift;
+      rem = s_rem;
+      const bool finished = s_h == rem;
+      __syncthreads();
+      if (finished) break;
+    }
+    if (tid == 0) s_cnt = 0u;
+    __syncthreads();
+    for (unsigned i = tid; i < m; i += T) {
+      const unsigned long long key = __ldcg(cand + i);
+      if ((key & mask) >= prefix) {
+        const unsigned p = atomicAdd(&s_cnt, 1u);
+        if (p < kk)
+          sk[p] = key;
+        else
+          atomicOr(err, kErrSelect);
+      }
+    }
+    __syncthreads();
+    for (int i = static_cast<int>(kk) + tid; i < n2; i += T) sk[i] = 0ull;
+    __syncthreads();
+    sort_desc(sk, n2);
+  }
   for (int r = tid; r < k; r += T) {
-    if (r < cnt) {
+    if (r < static_cast<int>(kk)) {
       const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(sk[r] & 0xFFFFFFFFull);
       out[r] = base + static_cast<long long>(pos);
     } else {
@@ -192,41 +220,28 @@ __global__ void __launch_bounds__(kSortThreads)
   }
 }
 
-int pass_grid(long long n) {
-  long long g = (n + 4095) / 4096;
-  if (g < 1) g = 1;
-  if (g > 608) g = 608;
-  return static_cast<int>(g);
-}
-
 }  // namespace
 
-cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, int k,
-                           cudaStream_t st) {
-  k_scan<<<1, kScanThreads, 0, st>>>(s.tile_counts, s.tile_offsets, n_tiles, s.state, k);
+cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, cudaStream_t st) {
+  k_scan<<<1, kScanThreads, 0, st>>>(s.tile_counts, s.tile_offsets, n_tiles, s.state);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (n_tiles > 0) k_scatter<<<static_cast<unsigned>(n_tiles), tile, 0, st>>>(s.masks, s.tile_offsets, s.rows, n);
   return cudaGetLastError();
 }
 
-cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk,
+cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk, int sms,
                         cudaStream_t st) {
-  const int g = pass_grid(n);
-  for (int p = 0; p < kRadixPasses; ++p) {
-    k_radix_pass<<<g, kPassThreads, 0, st>>>(s.keys, s.state, p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  k_gather<<<g, 256, 0, st>>>(s.keys, s.state, s.sel, s.err);
-  cudaError_t e = cudaGetLastError();
+  int cap = kSortMin;
+  while (cap < k) cap <<= 1;
+  const size_t smem = static_cast<size_t>(cap) * 8;
+  cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  int n2 = 1;
-  while (n2 < k) n2 <<= 1;
-  const size_t smem = static_cast<size_t>(n2) * 8;
-  e = cudaFuncSetAttribute(k_sort_out, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  k_sort_out<<<1, kSortThreads, smem, st>>>(s.state, s.sel, k, n2, index_base, out_topk);
+  long long g = (n + kTopkThreads * 8 - 1) / (kTopkThreads * 8);
+  if (g < 1) g = 1;
+  if (g > sms) g = sms;
+  k_topk<<<static_cast<unsigned>(g), kTopkThreads, smem, st>>>(s.keys, s.cand, s.state, k, cap, index_base,
+                                                              out_topk, s.err);
   return cudaGetLastError();
 }
 

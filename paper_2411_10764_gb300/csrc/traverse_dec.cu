@@ -1,0 +1,103 @@
+// Tree-walk kernels that build each candidate's features on chip from its
+// index (mixed-radix knob decode + feature program) instead of reading a
+// stored feature matrix, and the materialising decoder of mlt_decode_knobs.
+// ML^2Tuner Sec. 2: the explorer enumerates the search space of
+// configurations; Appendix A.2: the knobs are tiling sizes and virtual-thread
+// counts; Table 5: derived (hidden) features.
+#include "walk.cuh"
+
+namespace mlt {
+namespace {
+
+using namespace walk;
+
+using FullDecKernel = void (*)(TraverseArgs, DecodeParams);
+
+template <int G>
+FullDecKernel full_dec_kernel(int d) {
+  switch (d) {
+    case 1: return k_traverse_full_dec<1, G>;
+    case 2: return k_traverse_full_dec<2, G>;
+    case 3: return k_traverse_full_dec<3, G>;
+    case 4: return k_traverse_full_dec<4, G>;
+    case 5: return k_traverse_full_dec<5, G>;
+    case 6: return k_traverse_full_dec<6, G>;
+    case 7: return k_traverse_full_dec<7, G>;
+    case 8: return k_traverse_full_dec<8, G>;
+    case 9: return k_traverse_full_dec<9, G>;
+    case 10: return k_traverse_full_dec<10, G>;
+    default: return nullptr;
+  }
+}
+
+// One thread per candidate: decode into a shared-memory column, then write
+// the rows out coalesced.
+__global__ void __launch_bounds__(256)
+    k_decode_rows(const __grid_constant__ DecodeParams d, long long n, uint8_t* out_knobs, float* out_feats) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  float* xs = reinterpret_cast<float*>(smem);
+  const int TC = blockDim.x, tid = threadIdx.x, F = d.F;
+  const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  const int rows_here = static_cast<int>(min(static_cast<long long>(TC), n - tile0));
+  if (tid < rows_here) {
+    const long long idx = d.first_index + tile0 + tid;
+    decode_column(d, idx, xs, TC, tid);
+    if (out_knobs != nullptr) {
+      long long rem = idx;
+      for (int j = 0; j < d.n_knobs; ++j) {
+        const long long q = rem / d.radix[j];
+        out_knobs[(tile0 + tid) * d.n_knobs + j] = static_cast<uint8_t>(rem - q * d.radix[j]);
+        rem = q;
+      }
+    }
+  }
+  __syncthreads();
+  if (out_feats != nullptr) {
+    for (int v = tid; v < rows_here * F; v += TC) {
+      const int r = v / F;
+      const int f = v - r * F;
+      out_feats[(tile0 + r) * F + f] = xs[f * TC + r];
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, const DecodeParams& dec,
+                                const ScreenShape& shape, long long n_tiles, cudaStream_t st) {
+  if (n_tiles <= 0) return cudaSuccess;
+  const dim3 grid(static_cast<unsigned>(n_tiles)), block(shape.threads);
+  if (m.kind == kTableFull) {
+    FullDecKernel k = shape.group == 8   ? full_dec_kernel<8>(m.depth)
+                      : shape.group == 4 ? full_dec_kernel<4>(m.depth)
+                                         : full_dec_kernel<2>(m.depth);
+    if (k == nullptr) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(shape.smem));
+    if (e != cudaSuccess) return e;
+    k<<<grid, block, shape.smem, st>>>(args, dec);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact_dec<4>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(shape.smem));
+    if (e != cudaSuccess) return e;
+    k_traverse_compact_dec<4><<<grid, block, shape.smem, st>>>(args, dec);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* out_knobs, float* out_feats,
+                               cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  int tc = 256;
+  while (tc > 32 && static_cast<size_t>(dec.F) * tc * 4 > 200 * 1024) tc >>= 1;
+  const size_t smem = static_cast<size_t>(dec.F) * tc * 4;
+  cudaError_t e = cudaFuncSetAttribute(k_decode_rows, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const long long tiles = (n + tc - 1) / tc;
+  k_decode_rows<<<static_cast<unsigned>(tiles), tc, smem, st>>>(dec, n, out_knobs, out_feats);
+  return cudaGetLastError();
+}
+
+}  // namespace mlt

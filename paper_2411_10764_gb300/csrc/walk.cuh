@@ -1,0 +1,520 @@
+// Device code of the tree-ensemble walk (included by traverse.cu and
+// traverse_dec.cu, which instantiate the plain and the decoding kernels).
+//
+// ML^2Tuner (arXiv 2411.10764) Sec. 2: the configuration explorer scores
+// candidates with model V (validity) and model P (performance); Sec. 3 /
+// Table 3: both are XGBoost gbtree ensembles, so a prediction is the sum
+// over trees of the leaf each tree routes the feature vector to.
+//
+// Layout on chip (one CTA = one tile of TC candidates, one thread each):
+//   * the tile's features sit in shared memory transposed, [F][TC] fp32:
+//     thread c reads x[f] at f*TC + c, so its bank is c mod 32 whatever f
+//     is -- a warp gathering 32 different features of its 32 candidates is
+//     conflict-free;
+//   * full tables: trees stream through shared memory in chunks with
+//     cp.async.bulk (bulk TMA copies) completing on mbarriers, all warps of
+//     the CTA walking the same chunk; a thread walks G trees at once for
+//     instruction-level parallelism and adds their leaves in tree order, so
+//     the fp32 sum is exactly sequential over trees from 0.0f;
+//   * compact tables (deep, unbalanced trees): nodes are read from global
+//     memory through L1 (they do not fit a shared-memory chunk).
+#pragma once
+
+#include <cmath>
+
+#include "mlt_internal.cuh"
+
+namespace mlt {
+namespace walk {
+
+__host__ __device__ constexpr size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ---------------------------------------------------------------------------
+// mbarrier / bulk-copy helpers (inline PTX, sm_90+)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                              uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Wait for an mbarrier phase, giving up after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > kWaitLimitNs) return false;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Small math helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float sigmoid_f(float m) {
+  if (m >= 0.0f) return 1.0f / (1.0f + expf(-m));
+  const float e = expf(m);
+  return e / (1.0f + e);
+}
+
+// 64-bit rank key: larger key = better candidate.  High word: the score
+// mapped to an order-preserving unsigned integer (-0 folded onto +0); low
+// word: ~position, so equal scores rank the smaller position first.
+__device__ __forceinline__ unsigned long long make_key(float s, uint32_t pos) {
+  const uint32_t u = __float_as_uint(s == 0.0f ? 0.0f : s);
+  const uint32_t mono = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return (static_cast<unsigned long long>(mono) << 32) | (0xFFFFFFFFu - pos);
+}
+
+// Exact floor(log2 a) for a positive normal float, 0 otherwise.
+__device__ __forceinline__ float ilog2_exact(float a) {
+  const uint32_t u = __float_as_uint(a);
+  const uint32_t e = (u >> 23) & 0xFFu;
+  if ((u & 0x80000000u) || e == 0u || e == 0xFFu) return 0.0f;
+  return static_cast<float>(static_cast<int>(e) - 127);
+}
+
+// ---------------------------------------------------------------------------
+// Feature staging: thread c fills column c of xs[f*TC + c]
+// ---------------------------------------------------------------------------
+
+// One decoded candidate -> column c of the tile (mixed-radix digits, knob 0
+// least significant; then the feature program, one rounded op each).
+__device__ __forceinline__ bool decode_column(const DecodeParams& d, long long idx, float* xs, int TC,
+                                              int c) {
+  float kv[kMaxKnobs];
+  long long rem = idx;
+  for (int j = 0; j < d.n_knobs; ++j) {
+    const long long r = d.radix[j];
+    const long long q = rem / r;
+    const int digit = static_cast<int>(rem - q * r);
+    rem = q;
+    kv[j] = d.opts[d.opt_off[j] + digit];
+  }
+  bool nan = false;
+  const int nk = d.n_knobs;
+  for (int f = 0; f < d.F; ++f) {
+    const int sa = d.a[f], sb = d.b[f];
+    const float cf = d.c[f];
+    const float A = sa < 0 ? cf : (sa < nk ? kv[sa] : xs[(sa - nk) * TC + c]);
+    const float B = sb < 0 ? cf : (sb < nk ? kv[sb] : xs[(sb - nk) * TC + c]);
+    float x;
+    switch (d.op[f]) {
+      case 0: x = A; break;
+      case 1: x = ilog2_exact(A); break;
+      case 2: x = __fadd_rn(A, B); break;
+      case 3: x = __fsub_rn(A, B); break;
+      case 4: x = __fmul_rn(A, B); break;
+      case 5: x = __fdiv_rn(A, B); break;
+      case 6: x = ceilf(__fdiv_rn(A, B)); break;
+      case 7: x = __fsub_rn(A, __fmul_rn(B, floorf(__fdiv_rn(A, B)))); break;
+      case 8: x = (B < A) ? B : A; break;
+      case 9: x = (B > A) ? B : A; break;
+      case 10: x = (A > B) ? 1.0f : 0.0f; break;
+      default: x = (A == B) ? 1.0f : 0.0f; break;
+    }
+    nan |= (x != x);
+    xs[f * TC + c] = x;
+  }
+  return nan;
+}
+
+// Stage this thread's candidate (one row per thread: the 32 lanes of a
+// store hit 32 different banks).  Returns whether the row holds a NaN.
+__device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodeParams* dec, float* xs,
+                                          const uint32_t* rowidx, long long tile0, int rows_here,
+                                          int TC) {
+  const int F = a.F;
+  const int c = threadIdx.x;
+  if (c >= rows_here) {
+    for (int f = 0; f < F; ++f) xs[f * TC + c] = 0.0f;
+    return false;
+  }
+  const long long pos = a.p_pass ? static_cast<long long>(rowidx[c]) : tile0 + c;
+  if (dec != nullptr) return decode_column(*dec, dec->first_index + pos, xs, TC, c);
+  bool nan = false;
+  const float* src = a.feats + pos * F;
+  if (a.vec4) {
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    const int F4 = F >> 2;
+    constexpr int U = 4;
+    for (int q0 = 0; q0 < F4; q0 += U) {
+      float4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (q0 + u < F4) v[u] = __ldg(s4 + q0 + u);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (q0 + u < F4) {
+          const int f = (q0 + u) << 2;
+          xs[(f + 0) * TC + c] = v[u].x;
+          xs[(f + 1) * TC + c] = v[u].y;
+          xs[(f + 2) * TC + c] = v[u].z;
+          xs[(f + 3) * TC + c] = v[u].w;
+          nan |= (v[u].x != v[u].x) | (v[u].y != v[u].y) | (v[u].z != v[u].z) | (v[u].w != v[u].w);
+        }
+      }
+    }
+  } else {
+    for (int f = 0; f < F; ++f) {
+      const float x = __ldg(src + f);
+      xs[f * TC + c] = x;
+      nan |= (x != x);
+    }
+  }
+  return nan;
+}
+
+// ---------------------------------------------------------------------------
+// Epilogues
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_t* rowidx,
+                                            long long tile0, int rows_here, long long count, float acc) {
+  const int tid = threadIdx.x;
+  const bool in = tid < rows_here;
+  if (a.p_pass) {
+    if (in) {
+      const uint32_t pos = rowidx[tid];
+      a.out_perf[pos] = acc;
+      const unsigned long long key = make_key(acc, pos);
+      a.keys[tile0 + tid] = key;
+      atomicAdd(&a.hist[key >> (64 - kTopBits)], 1u);
+    }
+    return;
+  }
+  __shared__ unsigned warp_count[32];
+  const long long i = tile0 + tid;
+  const bool valid = in && (acc >= a.tau);
+  if (in) {
+    a.out_pvalid[i] = sigmoid_f(acc);
+    if (!valid) a.out_perf[i] = -INFINITY;
+  }
+  const unsigned ball = __ballot_sync(0xFFFFFFFFu, valid);
+  const int warp = tid >> 5;
+  if ((tid & 31) == 0) {
+    if (tile0 + warp * 32 < count) a.masks[(tile0 >> 5) + warp] = ball;
+    warp_count[warp] = __popc(ball);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    unsigned s = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += warp_count[w];
+    a.tile_counts[blockIdx.x] = s;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Full-table walk of one chunk of trees
+// ---------------------------------------------------------------------------
+// 32-bit shared-window loads.  `volatile` keeps them in program order with
+// the barriers and mbarrier waits around the walk; the walk below issues the
+// G trees' loads of one level back to back, so ordering costs no overlap.
+__device__ __forceinline__ uint2 lds_u2(uint32_t a) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ uint4 lds_u4(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ uint32_t lds_u32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ float lds_f32(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a));
+  return v;
+}
+
+// Go right?  x >= threshold; a missing x takes the node's default side.
+template <bool NANP>
+__device__ __forceinline__ uint32_t go_right(float x, uint32_t thr_bits, uint32_t meta) {
+  uint32_t right = x >= __uint_as_float(thr_bits) ? 1u : 0u;
+  if (NANP && (x != x) && !(meta >> 31)) right = 1u;
+  return right;
+}
+
+// Walk trees [0, nt) of the chunk at shared address tb; xa = shared address
+// of this thread's feature column (feature f at xa + f * row_bytes).  The
+// 32-bit product meta * row_bytes drops meta's bit 31 because row_bytes is a
+// multiple of 2.
+template <int D, int G, bool NANP>
+__device__ __forceinline__ float walk_chunk(uint32_t tb, int nt, uint32_t tree_bytes, uint32_t xa,
+                                            uint32_t row_bytes, float acc) {
+  constexpr FullLayout L = full_layout(D);
+  // byte offsets folded with the heap index of each region's first node
+  constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
+  constexpr uint32_t kMeta = L.off_meta - L.n_top * 4u;
+  constexpr uint32_t kLast = L.off_last - L.n_inner * 16u;
+  int t = 0;
+  for (; t + G <= nt; t += G) {
+    uint32_t base[G], j[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      base[g] = tb + static_cast<uint32_t>(t + g) * tree_bytes;
+      j[g] = 0;
+    }
+#pragma unroll
+    for (int l = 0; l < D - 1; ++l) {
+      uint32_t thr[G], meta[G];
+      if (l < static_cast<int>(L.top)) {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          const uint2 r = lds_u2(base[g] + j[g] * 8u);
+          thr[g] = r.x;
+          meta[g] = r.y;
+        }
+      } else {
+#pragma unroll
+        for (int g = 0; g < G; ++g) meta[g] = lds_u32(base[g] + kMeta + j[g] * 4u);
+#pragma unroll
+        for (int g = 0; g < G; ++g) thr[g] = lds_u32(base[g] + kThr + j[g] * 4u);
+      }
+      float x[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) x[g] = lds_f32(meta[g] * row_bytes + xa);
+#pragma unroll
+      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], thr[g], meta[g]);
+    }
+    uint4 r[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) r[g] = lds_u4(base[g] + kLast + j[g] * 16u);
+    float x[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+      acc += __uint_as_float(go_right<NANP>(x[g], r[g].x, r[g].y) ? r[g].w : r[g].z);
+  }
+  for (; t < nt; ++t) {
+    const uint32_t base = tb + static_cast<uint32_t>(t) * tree_bytes;
+    uint32_t j = 0;
+#pragma unroll
+    for (int l = 0; l < D - 1; ++l) {
+      uint32_t thr, meta;
+      if (l < static_cast<int>(L.top)) {
+        const uint2 r = lds_u2(base + j * 8u);
+        thr = r.x;
+        meta = r.y;
+      } else {
+        meta = lds_u32(base + kMeta + j * 4u);
+        thr = lds_u32(base + kThr + j * 4u);
+      }
+      const float x = lds_f32(meta * row_bytes + xa);
+      j = 2u * j + 1u + go_right<NANP>(x, thr, meta);
+    }
+    const uint4 r = lds_u4(base + kLast + j * 16u);
+    const float x = lds_f32(r.y * row_bytes + xa);
+    acc += __uint_as_float(go_right<NANP>(x, r.x, r.y) ? r.w : r.z);
+  }
+  return acc;
+}
+
+// Shared-memory layout of the full-table kernel (host and device agree):
+//   [0, feat) features [F][TC]; rows [TC] u32; nbuf chunk buffers; mbarriers.
+__host__ __device__ inline size_t full_smem_rows_off(int F, int TC) {
+  return align_up(static_cast<size_t>(F) * TC * 4, 128);
+}
+__host__ __device__ inline size_t full_smem_tbuf_off(int F, int TC) {
+  return full_smem_rows_off(F, TC) + align_up(static_cast<size_t>(TC) * 4, 128);
+}
+__host__ __device__ inline size_t full_smem_bytes(int F, int TC, int nbuf, uint32_t chunk_bytes) {
+  return align_up(full_smem_tbuf_off(F, TC) + static_cast<size_t>(nbuf) * chunk_bytes, 16) + 8 * 4;
+}
+
+template <int D, int G>
+__device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int TC = blockDim.x;
+  const int tid = threadIdx.x;
+  const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
+  if (tile0 >= count) return;  // whole CTA, before any copy is issued
+  const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
+
+  float* xs = reinterpret_cast<float*>(smem);
+  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + full_smem_rows_off(a.F, TC));
+  unsigned char* tbuf = smem + full_smem_tbuf_off(a.F, TC);
+  const uint32_t chunk_bytes = static_cast<uint32_t>(a.chunk_trees) * a.tree_bytes;
+  unsigned long long* bars = reinterpret_cast<unsigned long long*>(
+      smem + align_up(full_smem_tbuf_off(a.F, TC) + static_cast<size_t>(a.nbuf) * chunk_bytes, 16));
+  const int n_chunks = (a.n_trees + a.chunk_trees - 1) / a.chunk_trees;
+
+  if (tid == 0) {
+    for (int b = 0; b < a.nbuf; ++b) mbar_init(smem_u32(&bars[b]), 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  auto issue = [&](int c, int b) {
+    const int first = c * a.chunk_trees;
+    const int nt = min(a.chunk_trees, a.n_trees - first);
+    const uint32_t bytes = static_cast<uint32_t>(nt) * a.tree_bytes;
+    const uint32_t bar = smem_u32(&bars[b]);
+    mbar_expect_tx(bar, bytes);
+    bulk_copy_g2s(smem_u32(tbuf + static_cast<size_t>(b) * chunk_bytes),
+                  a.table + static_cast<size_t>(first) * a.tree_bytes, bytes, bar);
+  };
+  if (tid == 0)
+    for (int c = 0; c < a.nbuf && c < n_chunks; ++c) issue(c, c);
+
+  if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
+  // each thread stages its own row (and reads only its own rowidx entry)
+  const bool nan = __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+
+  float acc = 0.0f;
+  const uint32_t row_bytes = static_cast<uint32_t>(TC) * 4u;
+  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(tid) * 4u;
+  const uint32_t tbuf_a = smem_u32(tbuf);
+  for (int c = 0; c < n_chunks; ++c) {
+    const int b = c % a.nbuf;
+    const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(c / a.nbuf) & 1u);
+    if (!__syncthreads_and(ok)) {
+      if (tid == 0) {
+        // let every copy still in flight land before the CTA's shared memory
+        // is released, then report
+        for (int cc = c + 1; cc < n_chunks && cc < c + a.nbuf; ++cc)
+          mbar_wait_bounded(smem_u32(&bars[cc % a.nbuf]), static_cast<uint32_t>(cc / a.nbuf) & 1u);
+        mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(c / a.nbuf) & 1u);
+        atomicOr(a.err, kErrWaitTimeout);
+      }
+      return;
+    }
+    const uint32_t tb = tbuf_a + static_cast<uint32_t>(b) * chunk_bytes;
+    const int nt = min(a.chunk_trees, a.n_trees - c * a.chunk_trees);
+    acc = nan ? walk_chunk<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
+              : walk_chunk<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+    __syncthreads();
+    if (tid == 0 && c + a.nbuf < n_chunks) issue(c + a.nbuf, b);
+  }
+  finish_tile(a, rowidx, tile0, rows_here, count, acc);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(256) k_traverse_full(const __grid_constant__ TraverseArgs a) {
+  traverse_full_body<D, G>(a, nullptr);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(256)
+    k_traverse_full_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
+  traverse_full_body<D, G>(a, &d);
+}
+
+// ---------------------------------------------------------------------------
+// Compact-table walk (nodes from global memory)
+// ---------------------------------------------------------------------------
+__host__ __device__ inline size_t compact_smem_bytes(int F, int TC) {
+  return align_up(static_cast<size_t>(F) * TC * 4, 128) + align_up(static_cast<size_t>(TC) * 4, 128);
+}
+
+template <int G>
+__device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, const DecodeParams* dec) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int TC = blockDim.x;
+  const int tid = threadIdx.x;
+  const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
+  if (tile0 >= count) return;
+  const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
+
+  float* xs = reinterpret_cast<float*>(smem);
+  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + align_up(static_cast<size_t>(a.F) * TC * 4, 128));
+  if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
+  __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+
+  const uint32_t* offs = reinterpret_cast<const uint32_t*>(a.table);
+  const uint2* recs =
+      reinterpret_cast<const uint2*>(a.table + align_up(static_cast<size_t>(a.n_trees) * 4, 16));
+  float acc = 0.0f;
+  const int steps = a.max_depth + 1;
+  for (int t = 0; t < a.n_trees; t += G) {
+    const uint2* tr[G];
+    uint32_t j[G];
+    float leaf[G];
+    bool live[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      live[g] = (t + g) < a.n_trees;
+      tr[g] = recs + (live[g] ? __ldg(offs + t + g) : 0u);
+      j[g] = 0;
+      leaf[g] = 0.0f;
+    }
+    for (int s = 0; s < steps; ++s) {
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        if (!live[g]) continue;
+        const uint2 r = __ldg(tr[g] + j[g]);
+        if (r.y & kMetaLeaf) {
+          leaf[g] = __uint_as_float(r.x);
+          live[g] = false;
+        } else {
+          const float x = xs[(r.y & 0xFFFFu) * TC + tid];
+          uint32_t right = x >= __uint_as_float(r.x) ? 1u : 0u;
+          if ((x != x) && !(r.y & kMetaDefaultLeft)) right = 1u;
+          j[g] = ((r.y >> 16) & 0x3FFFu) + right;
+        }
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+      if (t + g < a.n_trees) acc += leaf[g];
+  }
+  finish_tile(a, rowidx, tile0, rows_here, count, acc);
+}
+
+template <int G>
+__global__ void __launch_bounds__(256) k_traverse_compact(const __grid_constant__ TraverseArgs a) {
+  traverse_compact_body<G>(a, nullptr);
+}
+
+template <int G>
+__global__ void __launch_bounds__(256)
+    k_traverse_compact_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
+  traverse_compact_body<G>(a, &d);
+}
+
+}  // namespace walk
+}  // namespace mlt

@@ -67,6 +67,7 @@ def lib(build_if_missing: bool = True):
             "mlt_last_survivor_count": [P, P],
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
+            "mlt_tune_shape": [i32, i32, i32, i32],
         }
         for name, args in sig.items():
             fn = getattr(L, name)
@@ -233,6 +234,11 @@ def phase_times():
     calls = C.c_int64()
     _check(lib().mlt_phase_times(out, 4, C.byref(calls)))
     return dict(zip(PHASES, [float(v) for v in out])), int(calls.value)
+
+
+def tune_shape(model_id: int, threads: int = 0, chunk_trees: int = 0, nbuf: int = 0) -> None:
+    """Fix (or with zeros, release) the walk's launch shape for one model."""
+    _check(lib().mlt_tune_shape(int(model_id), int(threads), int(chunk_trees), int(nbuf)))
 
 
 def kernel_launches() -> int:
