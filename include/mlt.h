@@ -139,6 +139,30 @@ int mlt_validity_cut(float thr, float *tau_out);
 int mlt_screen(void *stream, const float *feats, int64_t n, float thr, int k,
                float *out_pvalid, float *out_perf, int64_t *out_topk);
 
+/* mlt_screen for callers that cannot allocate device memory during a call:
+ * a process whose device memory is owned by another allocator (a
+ * framework's caching allocator, or a pool reserved up front), or a
+ * latency-critical loop that cannot afford cudaMalloc's implicit device
+ * synchronisation.  The paper has no counterpart; this is a property of the
+ * library only.  Same arguments, results and asynchrony as mlt_screen, but
+ * its scratch is a fixed array in the library's own device memory (about
+ * 5.1 MB, present on every GPU that loads the library until the process
+ * exits), so the call allocates nothing:
+ *   - n is limited to 262,144 candidates; a larger n returns MLT_EINVAL
+ *     before any GPU work;
+ *   - the first call on each device looks up the array's device address on
+ *     that device (make it the current device); issue that first call
+ *     before any stream capture;
+ *   - every call shares the one array: calls whose GPU work overlaps (for
+ *     example on two streams without ordering) race and give undefined
+ *     results;
+ *   - a device-side error bit (a bounded wait that gave up) lives in the
+ *     array too; it is cleared by the next call, and mlt_sync_status does
+ *     not report it.
+ * Models V and P must have been loaded with mlt_load_ensemble beforehand. */
+int mlt_screen_noalloc(void *stream, const float *feats, int64_t n, float thr, int k,
+                       float *out_pvalid, float *out_perf, int64_t *out_topk);
+
 /* mlt_screen with host buffers, for end-to-end use: copies feats_host
  * ([n][F] fp32) to the device, screens, and copies the three results back
  * into host buffers of the same shapes.  Synchronous on `stream`. */

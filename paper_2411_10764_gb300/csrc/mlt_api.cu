@@ -20,6 +20,27 @@
 #include "mlt.h"
 #include "mlt_internal.cuh"
 
+// Scratch of mlt_screen_noalloc: one fixed array in the module's global
+// memory (about 5.1 MB, held on every device that loads the library until
+// the process exits), carved into the same pieces the allocating path uses.
+namespace mlt_noalloc {
+constexpr long long kMaxN = 262144;  // candidates per call
+constexpr size_t align256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+constexpr size_t kWords = kMaxN / 32 + 8;  // warp ballots; tile counters (tiles hold >= 32)
+constexpr size_t kMasks = 0;
+constexpr size_t kCounts = align256(kMasks + kWords * 4);
+constexpr size_t kOffsets = align256(kCounts + kWords * 4);
+constexpr size_t kRows = align256(kOffsets + kWords * 4);
+constexpr size_t kKeys = align256(kRows + kMaxN * 4);
+constexpr size_t kCand = align256(kKeys + kMaxN * 8);
+constexpr size_t kState = align256(kCand + kMaxN * 8);
+constexpr size_t kErr = align256(kState + sizeof(mlt::SelectState));
+constexpr size_t kBytes = align256(kErr + sizeof(unsigned int));
+constexpr int kMaxDevices = 64;
+}  // namespace mlt_noalloc
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[mlt_noalloc::kBytes];
+
 namespace {
 
 using namespace mlt;
@@ -382,15 +403,15 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
   return MLT_OK;
 }
 
-// The whole screening sequence on `st` (caller holds g_mu).
-int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, long long n, float thr,
-               int k, float* out_pvalid, float* out_perf, int64_t* out_topk) {
+// The whole screening sequence on `st` with scratch `s` (caller holds g_mu).
+// `profile_ok`: phase events may be recorded.
+int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec, long long n, float thr,
+                    int k, float* out_pvalid, float* out_perf, int64_t* out_topk, const Scratch& s,
+                    bool profile_ok) {
   int dev = 0;
   int rc = current_device(&dev);
   if (rc != MLT_OK) return rc;
   rc = check_models(dev);
-  if (rc != MLT_OK) return rc;
-  rc = ensure_scratch(n);
   if (rc != MLT_OK) return rc;
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
@@ -398,7 +419,6 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   const ScreenShape sv = plan_for(V, g_F, n, g_shape[MLT_MODEL_V]);
   const ScreenShape sp = plan_for(P, g_F, (n + 1) / 2, g_shape[MLT_MODEL_P]);
   if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
-  const Scratch& s = g_scr.s;
   TraverseArgs a{};
   a.feats = feats;
   a.F = g_F;
@@ -425,7 +445,7 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   av.nbuf = sv.nbuf;
   av.max_depth = V.depth;
   cudaEvent_t* ev = nullptr;
-  if (g_profile) {
+  if (g_profile && profile_ok) {
     if (g_events_used + kPhases + 1 > g_events.size()) {
       for (int i = 0; i <= kPhases; ++i) {
         cudaEvent_t e;
@@ -460,6 +480,38 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
   g_launches += (tiles_v > 0 ? 1 : 0) + 1 + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
   return MLT_OK;
+}
+
+// Device address of g_noalloc_scratch on the current device, resolved the
+// first time per device (in host code the array's name is only a stand-in).
+unsigned char* g_noalloc_base[mlt_noalloc::kMaxDevices] = {};
+
+int noalloc_scratch(int dev, Scratch* out) {
+  using namespace mlt_noalloc;
+  if (dev < 0 || dev >= kMaxDevices) return fail(MLT_EINVAL, "device %d out of range for the static scratch", dev);
+  if (g_noalloc_base[dev] == nullptr) {
+    void* p = nullptr;
+    MLT_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch), "cudaGetSymbolAddress(static scratch)");
+    g_noalloc_base[dev] = static_cast<unsigned char*>(p);
+  }
+  unsigned char* b = g_noalloc_base[dev];
+  out->masks = reinterpret_cast<uint32_t*>(b + kMasks);
+  out->tile_counts = reinterpret_cast<uint32_t*>(b + kCounts);
+  out->tile_offsets = reinterpret_cast<uint32_t*>(b + kOffsets);
+  out->rows = reinterpret_cast<uint32_t*>(b + kRows);
+  out->keys = reinterpret_cast<unsigned long long*>(b + kKeys);
+  out->cand = reinterpret_cast<unsigned long long*>(b + kCand);
+  out->state = reinterpret_cast<SelectState*>(b + kState);
+  out->err = reinterpret_cast<unsigned int*>(b + kErr);
+  return MLT_OK;
+}
+
+// The screening sequence with the library's own (allocated) scratch.
+int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, long long n, float thr, int k,
+               float* out_pvalid, float* out_perf, int64_t* out_topk) {
+  const int rc = ensure_scratch(n);
+  if (rc != MLT_OK) return rc;
+  return run_screen_with(st, feats, dec, n, thr, k, out_pvalid, out_perf, out_topk, g_scr.s, true);
 }
 
 }  // namespace
@@ -535,6 +587,30 @@ int mlt_screen(void* stream, const float* feats, int64_t n, float thr, int k, fl
   std::lock_guard<std::mutex> lk(g_mu);
   if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
   return run_screen(static_cast<cudaStream_t>(stream), feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk);
+}
+
+int mlt_screen_noalloc(void* stream, const float* feats, int64_t n, float thr, int k, float* out_pvalid,
+                       float* out_perf, int64_t* out_topk) {
+  int rc = check_screen_args(n, thr, k);
+  if (rc != MLT_OK) return rc;
+  if (n > mlt_noalloc::kMaxN)
+    return fail(MLT_EINVAL, "n=%lld exceeds the %lld candidates the static scratch holds", static_cast<long long>(n),
+                mlt_noalloc::kMaxN);
+  if ((n > 0 && (feats == nullptr || out_pvalid == nullptr || out_perf == nullptr)) || out_topk == nullptr)
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  int dev = 0;
+  rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  Scratch s;
+  rc = noalloc_scratch(dev, &s);
+  if (rc != MLT_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // the array keeps the previous call's contents: the error word must start
+  // at zero (every other piece is rewritten before it is read)
+  MLT_CUDA(cudaMemsetAsync(s.err, 0, sizeof(unsigned int), st), "clear static error word");
+  return run_screen_with(st, feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk, s, false);
 }
 
 int mlt_screen_decoded(void* stream, const int32_t* radices, const float* option_values, int n_knobs,

@@ -68,6 +68,7 @@ def lib(build_if_missing: bool = True):
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_shape": [i32, i32, i32, i32],
+            "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
         }
         for name, args in sig.items():
             fn = getattr(L, name)
@@ -159,6 +160,21 @@ def screen(feats, thr: float, k: int, out_pvalid=None, out_perf=None, out_topk=N
     pv, pf, tk = _outputs(n, k, feats.device, out_pvalid, out_perf, out_topk)
     _check(lib().mlt_screen(_stream_ptr(stream), _dptr(feats), n, C.c_float(thr), int(k),
                             _dptr(pv), _dptr(pf), _dptr(tk)))
+    return pv, pf, tk
+
+
+def screen_noalloc(feats, thr: float, k: int, out_pvalid=None, out_perf=None, out_topk=None,
+                   stream=None):
+    """mlt_screen_noalloc: like screen(), with the library's fixed scratch
+    (n <= 262,144; overlapping calls race)."""
+    import torch
+
+    if not (isinstance(feats, torch.Tensor) and feats.is_cuda and feats.dtype == torch.float32):
+        raise TypeError("feats must be a float32 CUDA tensor")
+    n = feats.shape[0]
+    pv, pf, tk = _outputs(n, k, feats.device, out_pvalid, out_perf, out_topk)
+    _check(lib().mlt_screen_noalloc(_stream_ptr(stream), _dptr(feats), n, C.c_float(thr), int(k),
+                                    _dptr(pv), _dptr(pf), _dptr(tk)))
     return pv, pf, tk
 
 
