@@ -238,7 +238,6 @@ def run_ours(args):
     if sampler:
         sampler.start()
     launches0 = mlt.kernel_launches()
-    mlt.profile_phases(True)
     wall0 = time.perf_counter()
     for i in range(args.steps):
         flush.fill_(float(i))
@@ -251,6 +250,15 @@ def run_ours(args):
         dist.barrier()
     clocks = sampler.stop() if sampler else None
     launches = mlt.kernel_launches() - launches0
+    mlt.sync_status(stream)
+    # per-phase device times: a second pass of the same steps with the
+    # library's phase events on the same stream (kept out of the timed pass:
+    # events between kernels stop one kernel's launch from overlapping the
+    # previous kernel's tail)
+    mlt.profile_phases(True)
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        step()
     phases, calls = mlt.phase_times()
     mlt.profile_phases(False)
     mlt.sync_status(stream)
@@ -319,6 +327,7 @@ def run_ours(args):
         "config": dict(config_dict(w), seed=args.seed, parallelism=f"replicas x{world}"),
         "survivors": survivors,
         "phases_ms": {kk: vv / max(calls, 1) for kk, vv in phases.items()},
+        "phases_note": "second pass of the same steps with CUDA events between phases",
         "roofline": {
             "bound": "alu", "kernel": f"{dominant} (tree walk)",
             "achieved": achieved / 1e9, "peak": visit_peak / 1e9, "unit": "Gvisit/s",

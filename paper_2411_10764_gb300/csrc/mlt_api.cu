@@ -433,6 +433,8 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   a.tile_counts = s.tile_counts;
   a.keys = s.keys;
   a.hist = s.state->hist;
+  a.tile_offsets = s.tile_offsets;
+  a.state_rw = s.state;
   a.err = s.err;
   a.decode = dec != nullptr;
 
@@ -478,7 +480,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   if (ev) MLT_CUDA(cudaEventRecord(ev[3], st), "cudaEventRecord");
   MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, sm_count(), st), "top-k launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
-  g_launches += (tiles_v > 0 ? 1 : 0) + 1 + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
+  g_launches += (tiles_v > 0 ? 1 : 0) + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
   return MLT_OK;
 }
 

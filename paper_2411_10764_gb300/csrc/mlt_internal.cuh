@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 #include <cuda_runtime.h>
 
 namespace mlt {
@@ -115,8 +116,8 @@ struct SelectState {
   unsigned int survivors;  // valid candidates of the current batch
   unsigned int n_cand;     // keys collected for the final sort
   unsigned int ticket;     // CTAs of the top-k kernel that finished
-  unsigned int pad;
-  unsigned int hist[kTopBins];
+  unsigned int v_ticket;   // CTAs of the V pass that finished
+  unsigned int hist[kTopBins];  // 16-byte aligned
 };
 
 struct Scratch {
@@ -134,6 +135,8 @@ struct Scratch {
 // Launch descriptors
 // ---------------------------------------------------------------------------
 struct TraverseArgs {
+  uint32_t* tile_offsets;  // V pass: exclusive prefix of tile_counts (last CTA)
+  SelectState* state_rw;   // V pass: written by the last CTA
   // candidates
   const float* feats;      // [n][F] (null when decoding)
   int F;
@@ -190,6 +193,31 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args,
                                 long long n_tiles, cudaStream_t st);
 cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* out_knobs,
                                float* out_feats, cudaStream_t st);
+
+// Launch with programmatic dependent launch allowed: the kernel may start
+// while the previous kernel on the stream finishes; it must execute
+// pdl_wait() before it touches anything that kernel (or any earlier one)
+// writes, and pdl_trigger() once its own dependents may be scheduled.
+template <typename... K, typename... A>
+cudaError_t launch_pdl(void (*kernel)(K...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       A&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<A>(args)...);
+}
+
+#ifdef __CUDACC__
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+#endif
 
 // select.cu
 cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles,

@@ -20,43 +20,14 @@
 namespace mlt {
 namespace {
 
-constexpr int kScanThreads = 1024;
 constexpr int kTopkThreads = 512;
 constexpr int kSortMin = 8192;  // sort buffer entries (at least pow2(k))
-
-__global__ void __launch_bounds__(kScanThreads)
-    k_scan(const uint32_t* counts, uint32_t* offsets, long long n_tiles, SelectState* st) {
-  __shared__ unsigned part[kScanThreads];
-  const int T = blockDim.x, tid = threadIdx.x;
-  const long long per = (n_tiles + T - 1) / T;
-  const long long b = tid * per;
-  const long long e = min(n_tiles, b + per);
-  unsigned s = 0;
-  for (long long i = b; i < e; ++i) s += counts[i];
-  part[tid] = s;
-  __syncthreads();
-  for (int off = 1; off < T; off <<= 1) {
-    const unsigned v = tid >= off ? part[tid - off] : 0u;
-    __syncthreads();
-    part[tid] += v;
-    __syncthreads();
-  }
-  unsigned run = part[tid] - s;
-  for (long long i = b; i < e; ++i) {
-    offsets[i] = run;
-    run += counts[i];
-  }
-  if (tid == T - 1) {
-    st->survivors = part[T - 1];
-    st->n_cand = 0u;
-    st->ticket = 0u;
-  }
-  for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
-}
 
 __global__ void __launch_bounds__(256)
     k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n) {
   __shared__ unsigned wc[32];
+  pdl_wait();
+  pdl_trigger();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const long long tile0 = static_cast<long long>(blockIdx.x) * blockDim.x;
   const long long first = tile0 + warp * 32;
@@ -92,33 +63,40 @@ __global__ void __launch_bounds__(kTopkThreads)
     k_topk(const unsigned long long* keys, unsigned long long* cand, SelectState* st, int k, int cap,
            long long base, int64_t* out, unsigned* err) {
   extern __shared__ __align__(16) unsigned long long sk[];  // cap entries
-  __shared__ unsigned part[kTopkThreads];
+  __shared__ unsigned warp_sum[kTopkThreads / 32];
   __shared__ unsigned s_bin, s_last, s_digit, s_rem, s_h, s_cnt;
   __shared__ unsigned h256[256];
-  const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31;
+  pdl_wait();
+  const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned S = st->survivors;
   const unsigned kk = S < static_cast<unsigned>(k) ? S : static_cast<unsigned>(k);
 
-  // 1. bucket of the kk-th largest key: thread t owns the top bins
-  //    [nb-1-t*per, nb-1-(t+1)*per+1], scanned from the top
-  constexpr int per = kTopBins / kTopkThreads;
+  // 1. bucket of the kk-th largest key.  Thread t holds the 8 bins
+  //    [4096-8(t+1), 4096-8t) in registers; threads are ordered from the top
+  //    bins down, so an exclusive scan over threads counts the keys above.
+  constexpr int per = kTopBins / kTopkThreads;  // 8
+  static_assert(per == 8, "two uint4 loads per thread");
+  const uint4* h4 = reinterpret_cast<const uint4*>(st->hist + (kTopBins - per * (tid + 1)));
+  const uint4 lo4 = __ldcg(h4), hi4 = __ldcg(h4 + 1);
+  const unsigned hb[per] = {hi4.w, hi4.z, hi4.y, hi4.x, lo4.w, lo4.z, lo4.y, lo4.x};  // descending bins
   unsigned local = 0;
-  for (int q = 0; q < per; ++q) local += st->hist[kTopBins - 1 - (tid * per + q)];
-  part[tid] = local;
+#pragma unroll
+  for (int q = 0; q < per; ++q) local += hb[q];
+  unsigned x = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sum[warp] = x;
   if (tid == 0) s_bin = kTopBins;  // nothing to select unless found
   __syncthreads();
-  for (int off = 1; off < T; off <<= 1) {
-    const unsigned v = tid >= off ? part[tid - off] : 0u;
-    __syncthreads();
-    part[tid] += v;
-    __syncthreads();
-  }
-  unsigned above = part[tid] - local;
+  unsigned above = x - local;
+  for (int w = 0; w < warp; ++w) above += warp_sum[w];
+#pragma unroll
   for (int q = 0; q < per; ++q) {
-    const int b = kTopBins - 1 - (tid * per + q);
-    const unsigned h = st->hist[b];
-    if (kk > 0 && above < kk && kk <= above + h) s_bin = static_cast<unsigned>(b);
-    above += h;
+    if (kk > 0 && above < kk && kk <= above + hb[q]) s_bin = static_cast<unsigned>(kTopBins - 1 - (tid * per + q));
+    above += hb[q];
   }
   __syncthreads();
   const unsigned long long bin = s_bin;
@@ -150,6 +128,7 @@ __global__ void __launch_bounds__(kTopkThreads)
   if (!s_last) return;
   __threadfence();
   const unsigned m = *reinterpret_cast<volatile unsigned*>(&st->n_cand);
+  if (tid == 0) st->v_ticket = 0u;  // in case a V pass ended early
   int n2 = 1;
   while (n2 < static_cast<int>(kk)) n2 <<= 1;
   if (m <= static_cast<unsigned>(cap)) {
@@ -223,11 +202,12 @@ __global__ void __launch_bounds__(kTopkThreads)
 }  // namespace
 
 cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, cudaStream_t st) {
-  k_scan<<<1, kScanThreads, 0, st>>>(s.tile_counts, s.tile_offsets, n_tiles, s.state);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  if (n_tiles > 0) k_scatter<<<static_cast<unsigned>(n_tiles), tile, 0, st>>>(s.masks, s.tile_offsets, s.rows, n);
-  return cudaGetLastError();
+  if (n_tiles <= 0) {
+    // no V pass ran: start the selection state from zero survivors
+    return cudaMemsetAsync(s.state, 0, sizeof(SelectState), st);
+  }
+  return launch_pdl(k_scatter, dim3(static_cast<unsigned>(n_tiles)), dim3(tile), 0, st, s.masks,
+                    static_cast<const uint32_t*>(s.tile_offsets), s.rows, n);
 }
 
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk, int sms,
@@ -237,12 +217,12 @@ cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_ba
   const size_t smem = static_cast<size_t>(cap) * 8;
   cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  long long g = (n + kTopkThreads * 8 - 1) / (kTopkThreads * 8);
+  long long g = (n + 1023) / 1024;  // about one pass of the collection loop per warp
   if (g < 1) g = 1;
-  if (g > sms) g = sms;
-  k_topk<<<static_cast<unsigned>(g), kTopkThreads, smem, st>>>(s.keys, s.cand, s.state, k, cap, index_base,
-                                                              out_topk, s.err);
-  return cudaGetLastError();
+  if (g > 4LL * sms) g = 4LL * sms;
+  return launch_pdl(k_topk, dim3(static_cast<unsigned>(g)), dim3(kTopkThreads), smem, st,
+                    static_cast<const unsigned long long*>(s.keys), s.cand, s.state, k, cap, index_base, out_topk,
+                    s.err);
 }
 
 }  // namespace mlt

@@ -13,7 +13,7 @@ using namespace walk;
 
 constexpr size_t kSmPerSm = 228 * 1024;  // shared memory per SM
 constexpr size_t kCtaReserve = 1024;     // reserved per resident CTA
-constexpr size_t kStaticSmem = 128;      // finish_tile's warp counters
+constexpr size_t kStaticSmem = 512;      // finish_tile and scan_tiles statics
 
 using FullKernel = void (*)(TraverseArgs);
 
@@ -126,12 +126,14 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    k<<<grid, block, shape.smem, st>>>(args);
+    e = launch_pdl(k, grid, block, shape.smem, st, args);
+    if (e != cudaSuccess) return e;
   } else {
     cudaError_t e = cudaFuncSetAttribute(k_traverse_compact<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    k_traverse_compact<4><<<grid, block, shape.smem, st>>>(args);
+    e = launch_pdl(k_traverse_compact<4>, grid, block, shape.smem, st, args);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

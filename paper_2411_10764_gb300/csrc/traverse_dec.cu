@@ -75,13 +75,15 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    k<<<grid, block, shape.smem, st>>>(args, dec);
+    e = launch_pdl(k, grid, block, shape.smem, st, args, dec);
+    if (e != cudaSuccess) return e;
   } else {
     cudaError_t e = cudaFuncSetAttribute(k_traverse_compact_dec<4>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    k_traverse_compact_dec<4><<<grid, block, shape.smem, st>>>(args, dec);
+    e = launch_pdl(k_traverse_compact_dec<4>, grid, block, shape.smem, st, args, dec);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

@@ -207,18 +207,59 @@ __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodePar
 // ---------------------------------------------------------------------------
 // Epilogues
 // ---------------------------------------------------------------------------
+
+// Exclusive scan of the per-tile survivor counts by one CTA, then the
+// survivor total and a fresh selection state for the P pass and top-k.
+__device__ __forceinline__ void scan_tiles(const uint32_t* counts, uint32_t* offsets, long long n_tiles,
+                                           SelectState* st) {
+  __shared__ unsigned warp_sum[32];
+  __shared__ unsigned carry;
+  const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = T >> 5;
+  if (tid == 0) carry = 0;
+  __syncthreads();
+  for (long long base = 0; base < n_tiles; base += T) {
+    const long long i = base + tid;
+    const unsigned v = i < n_tiles ? __ldcg(counts + i) : 0u;
+    unsigned x = v;  // inclusive warp scan
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sum[warp] = x;
+    __syncthreads();
+    unsigned before = carry;
+    for (int w = 0; w < warp; ++w) before += warp_sum[w];
+    if (i < n_tiles) offsets[i] = before + x - v;
+    __syncthreads();
+    if (tid == T - 1) carry = before + x;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    st->survivors = carry;
+    st->n_cand = 0u;
+    st->ticket = 0u;
+    st->v_ticket = 0u;
+  }
+  for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
+  (void)nw;
+}
 __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_t* rowidx,
                                             long long tile0, int rows_here, long long count, float acc) {
   const int tid = threadIdx.x;
   const bool in = tid < rows_here;
   if (a.p_pass) {
+    unsigned bin = 0xFFFFFFFFu;
     if (in) {
       const uint32_t pos = rowidx[tid];
       a.out_perf[pos] = acc;
       const unsigned long long key = make_key(acc, pos);
       a.keys[tile0 + tid] = key;
-      atomicAdd(&a.hist[key >> (64 - kTopBits)], 1u);
+      bin = static_cast<unsigned>(key >> (64 - kTopBits));
     }
+    // one atomic per distinct bucket of the warp
+    const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin);
+    if (in && (tid & 31) == __ffs(peers) - 1) atomicAdd(&a.hist[bin], static_cast<unsigned>(__popc(peers)));
     return;
   }
   __shared__ unsigned warp_count[32];
@@ -234,11 +275,21 @@ __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_
     if (tile0 + warp * 32 < count) a.masks[(tile0 >> 5) + warp] = ball;
     warp_count[warp] = __popc(ball);
   }
+  __shared__ unsigned is_last;
   __syncthreads();
   if (tid == 0) {
     unsigned s = 0;
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += warp_count[w];
     a.tile_counts[blockIdx.x] = s;
+    __threadfence();
+    is_last = atomicAdd(&a.state_rw->v_ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (is_last) {
+    // the last V tile to finish turns the tile counts into offsets and
+    // resets the selection state (no CTA waits for another)
+    __threadfence();
+    scan_tiles(a.tile_counts, a.tile_offsets, gridDim.x, a.state_rw);
   }
 }
 
@@ -371,6 +422,9 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   const int TC = blockDim.x;
   const int tid = threadIdx.x;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  // the P pass needs the survivor count of the kernels before it; the V
+  // pass only needs them before it reads the features
+  if (a.p_pass) pdl_wait();
   const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
   if (tile0 >= count) return;  // whole CTA, before any copy is issued
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
@@ -398,8 +452,9 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
                   a.table + static_cast<size_t>(first) * a.tree_bytes, bytes, bar);
   };
   if (tid == 0)
-    for (int c = 0; c < a.nbuf && c < n_chunks; ++c) issue(c, c);
+    for (int c = 0; c < a.nbuf && c < n_chunks; ++c) issue(c, c);  // tables are static
 
+  if (!a.p_pass) pdl_wait();
   if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
   // each thread stages its own row (and reads only its own rowidx entry)
   const bool nan = __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
@@ -429,6 +484,7 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     __syncthreads();
     if (tid == 0 && c + a.nbuf < n_chunks) issue(c + a.nbuf, b);
   }
+  pdl_trigger();
   finish_tile(a, rowidx, tile0, rows_here, count, acc);
 }
 
@@ -456,6 +512,7 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
   const int TC = blockDim.x;
   const int tid = threadIdx.x;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  pdl_wait();
   const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
   if (tile0 >= count) return;
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
@@ -502,6 +559,7 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
     for (int g = 0; g < G; ++g)
       if (t + g < a.n_trees) acc += leaf[g];
   }
+  pdl_trigger();
   finish_tile(a, rowidx, tile0, rows_here, count, acc);
 }
 
