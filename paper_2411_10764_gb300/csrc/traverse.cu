@@ -37,50 +37,62 @@ FullKernel full_kernel(int d) {
 }  // namespace
 
 // Choose candidates per CTA (threads), trees per shared-memory chunk, chunk
-// buffers and trees walked together (group) for a full table.  The cost of
-// an option is the busiest SM's walking time: its candidates times the node
-// visits per candidate, slowed down when too few independent walks are in
-// flight to hide shared-memory latency, or the tree-streaming time if that
-// is longer (tables are re-streamed once per CTA).
+// buffers and trees walked together (group) for a full table.  Rules (from
+// sweeps of every shape on the five workloads):
+//   * every CTA re-streams the whole table through shared memory, and with
+//     small CTAs the stream (not the walk) sets the pace, so CTAs hold 256
+//     candidates unless the batch would then occupy fewer than a quarter of
+//     the SMs; then the largest size that reaches that is used;
+//   * when the busiest SM holds two or more tiles, a shape that keeps two
+//     CTAs resident (twice the warps to hide shared-memory latency) beats
+//     one CTA with bigger chunks: take the largest chunk that still allows
+//     two; otherwise one CTA with the largest chunk (fewest barriers);
+//   * a thread walks 8 trees at once when 8 warps or fewer share the SM,
+//     else 4 (the chunk permitting).
 ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms, int optin,
                       const ShapeOverride& ov) {
-  ScreenShape best{};
-  double best_cost = 1e300;
   if (sms < 1) sms = 1;
   if (n_eff < 1) n_eff = 1;
-  for (int tc : {256, 128, 64, 32}) {
-    if (ov.threads && tc != ov.threads) continue;
-    for (int ch : {16, 8, 4, 2, 1}) {
-      if (ov.chunk_trees && ch != ov.chunk_trees) continue;
-      if (ch > n_trees && ch != 1 && !(ch / 2 < n_trees)) continue;
-      const int chunk = std::min(ch, n_trees);
-      for (int nb : {2, 3}) {
-        if (ov.nbuf && nb != ov.nbuf) continue;
-        const size_t smem = full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb);
-        if (smem + kStaticSmem > static_cast<size_t>(optin)) continue;
-        const int ctas_sm = static_cast<int>(std::min<size_t>(
-            {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / tc), 32}));
-        if (ctas_sm < 1) continue;
-        const long long tiles = (n_eff + tc - 1) / tc;
-        const long long tiles_sm = (tiles + sms - 1) / sms;
-        const int resident = static_cast<int>(std::min<long long>(ctas_sm, tiles_sm));
-        const int warps = resident * tc / 32;
+  auto smem_of = [&](int tc, int chunk, int nb) {
+    return full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb);
+  };
+  auto fits = [&](size_t smem) { return smem + kStaticSmem <= static_cast<size_t>(optin); };
+  auto resident = [&](size_t smem, int tc) {
+    return static_cast<int>(std::min<size_t>(
+        {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / tc), 32}));
+  };
+  int tc = 256;
+  if (!ov.threads) {
+    while (tc > 32 && (n_eff + tc - 1) / tc < (sms + 3) / 4) tc >>= 1;
+  } else {
+    tc = ov.threads;
+  }
+  const long long tiles = (n_eff + tc - 1) / tc;
+  const long long tiles_sm = (tiles + sms - 1) / sms;
+  ScreenShape best{};
+  int best_rank = -1;
+  for (int ch : {16, 8, 4, 2, 1}) {
+    if (ov.chunk_trees && ch != ov.chunk_trees) continue;
+    const int chunk = std::min(ch, n_trees);
+    for (int nb : {2, 3}) {
+      if (ov.nbuf && nb != ov.nbuf) continue;
+      const size_t smem = smem_of(tc, chunk, nb);
+      if (!fits(smem)) continue;
+      const int res = std::min<long long>(resident(smem, tc), tiles_sm);
+      // rank: two resident CTAs when there are two tiles to run, then
+      // chunk size, then fewer buffers
+      const int want2 = tiles_sm >= 2 && res >= 2 ? 1 : 0;
+      const int rank = want2 * 1000 + chunk * 10 + (3 - nb);
+      if (rank > best_rank) {
+        best_rank = rank;
+        const int warps = res * tc / 32;
         int group = warps <= 8 ? 8 : 4;
-        group = std::min(group, std::max(2, chunk >= 8 ? 8 : chunk >= 4 ? 4 : 2));
-        const double chains = static_cast<double>(warps) * std::min(group, chunk);
-        const double eff = std::min(1.0, chains / 64.0);
-        const double walk = tc * 0.11 / eff * (1.0 + 0.5 / chunk);   // per tree per depth level
-        const double stream = static_cast<double>(tb) / 127.0;        // per tree, cycles
-        const double cost = static_cast<double>(tiles_sm) * std::max(walk * 8.0, stream) +
-                            1e-6 * nb;  // fewer buffers on ties
-        if (cost < best_cost) {
-          best_cost = cost;
-          best.threads = tc;
-          best.chunk_trees = chunk;
-          best.nbuf = nb;
-          best.group = group;
-          best.smem = smem;
-        }
+        group = std::min(group, chunk >= 8 ? 8 : chunk >= 4 ? 4 : 2);
+        best.threads = tc;
+        best.chunk_trees = chunk;
+        best.nbuf = nb;
+        best.group = group;
+        best.smem = smem;
       }
     }
   }
