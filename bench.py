@@ -171,6 +171,36 @@ def config_dict(w):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
+def library_source_hash() -> str:
+    """Hash of the CUDA sources and the C header (order as in the profiles)."""
+    import glob
+    import hashlib
+
+    csrc = os.path.join(ROOT, "paper_2411_10764_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "*.cu"))) + sorted(glob.glob(os.path.join(csrc, "*.cuh")))
+    files.append(os.path.join(ROOT, "include", "mlt.h"))
+    h = hashlib.sha256()
+    for path in files:
+        with open(path, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def dram_traffic(config: int, phase: str):
+    """DRAM bytes per launch of the phase's kernel from the committed ncu
+    capture, or None if there is none or the kernels changed since."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            tr = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if tr.get("source_hash") != library_source_hash():
+        return None
+    ent = tr.get(f"config{config}:{phase}")
+    return ent.get("dram_bytes_per_launch") if ent else None
+
+
 def algorithmic_counts(w, survivors):
     """Node visits and algorithmic HBM bytes of one step (see the design notes)."""
     c = w.cfg
@@ -309,16 +339,7 @@ def run_ours(args):
     dom_bytes = (cnt["feat_bytes"] + cnt["v_table_bytes"]) if dominant == "v_pass" else \
         (cnt["survivor_feat_bytes"] + cnt["p_table_bytes"])
     step_bytes = cnt["feat_bytes"] + cnt["v_table_bytes"] + cnt["p_table_bytes"]
-    traffic = None
-    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tr_path):
-        try:
-            with open(tr_path) as f:
-                tr = json.load(f)
-            ent = tr.get(f"config{args.config}:{dominant}")
-            traffic = ent.get("dram_bytes_per_launch") if ent else None
-        except (OSError, ValueError):
-            traffic = None
+    traffic = dram_traffic(args.config, dominant)
     line = {
         "metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
