@@ -102,7 +102,7 @@ int mlt_set_num_features(int F);
  *   model_id : MLT_MODEL_V, MLT_MODEL_P or MLT_MODEL_A
  *   nodes    : host array of n_trees * (2^(depth+1)-1) heap-order slots;
  *              the caller keeps ownership (it is only read during the call)
- *   n_trees  : 1 .. 65536;  depth : 1 .. 12
+ *   n_trees  : 1 .. 65536;  depth : 1 .. 14
  * Validation (MLT_EINVAL): slot 0 is a split or a leaf; every split's two
  * children are splits or leaves; slots at `depth` that are reachable are
  * leaves; split features lie in [0, F); thresholds and leaves are finite;
@@ -168,6 +168,24 @@ int mlt_screen_noalloc(void *stream, const float *feats, int64_t n, float thr, i
  * into host buffers of the same shapes.  Synchronous on `stream`. */
 int mlt_screen_host(void *stream, const float *feats_host, int64_t n, float thr, int k,
                     float *pvalid_host, float *perf_host, int64_t *topk_host);
+
+/* Model A rerank (Sec. 2, "Hidden Feature Extractor & ML Model A"): from the
+ * (alpha+1)N candidates kept by screening, model A -- a performance
+ * regressor over visible and hidden features, typically deeper than P
+ * (depth 14 in Table 3) -- selects the final N:
+ *   out_score[i] = margin_A(row cand[i] of feats) (fp32, tree order) for
+ *                  0 <= cand[i] < n; -infinity for cand[i] < 0 (an empty
+ *                  slot, e.g. the -1 padding of out_topk);
+ *   out_final[r] = the r-th entry of cand by (score descending, candidate
+ *                  index ascending), r < n_final; -1 past the valid entries.
+ * Arguments:
+ *   feats      device [n][F] fp32, the same matrix the candidates index
+ *   cand       device [m] int64 (typically mlt_screen's out_topk), 0 <= m <= 16384
+ *   n_final    1 .. 16384;  out_score device [m] fp32;  out_final device [n_final] int64
+ * Needs model A loaded with the current F.  An index >= n is scored -inf and
+ * reported by the next mlt_sync_status (MLT_EINVAL).  Asynchronous. */
+int mlt_rerank(void *stream, const float *feats, int64_t n, const int64_t *cand, int m,
+               int n_final, float *out_score, int64_t *out_final);
 
 /* Decode candidate indices into knob choices and build their features
  * (the explorer's enumeration of the search space, Sec. 2; knobs are tiling

@@ -11,6 +11,7 @@ from .oracle import (  # noqa: F401
     decode,
     features,
     margins,
+    rerank,
     screen,
     screen_rows,
     sigmoid,

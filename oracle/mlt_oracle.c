@@ -261,6 +261,42 @@ int64_t orc_screen(const float *feats, int64_t n, int F,
 }
 
 /* ------------------------------------------------------------------ */
+/* Model A rerank (Sec. 2 "Hidden Feature Extractor & ML Model A")     */
+/* ------------------------------------------------------------------ */
+
+/* From the kept candidates cand[0..m), model A -- a performance regressor
+ * over visible and hidden features -- selects the final n_final:
+ *   out_score[i] = margin_A(feats row cand[i]) for cand[i] >= 0, -inf else;
+ *   out_final    = the n_final entries of cand with the highest score, equal
+ *                  scores by the smaller candidate index, -1 padded.
+ * Returns the number of valid entries, or -1 on allocation failure. */
+int64_t orc_rerank(const float *feats, int F, const int64_t *cand, int64_t m,
+                   const orc_node *a_nodes, int a_trees, int a_depth, int n_final,
+                   float *out_score, int64_t *out_final)
+{
+    scored *all = (scored *)malloc((size_t)(m > 0 ? m : 1) * sizeof(scored));
+    if (!all)
+        return -1;
+    int64_t v = 0;
+    for (int64_t i = 0; i < m; ++i) {
+        if (cand[i] < 0) {
+            out_score[i] = -INFINITY;
+            continue;
+        }
+        float s = orc_margin(a_nodes, a_trees, a_depth, feats + cand[i] * (int64_t)F);
+        out_score[i] = s;
+        all[v].score = s;
+        all[v].index = cand[i];
+        ++v;
+    }
+    qsort(all, (size_t)v, sizeof(scored), by_score_desc_index_asc);
+    for (int r = 0; r < n_final; ++r)
+        out_final[r] = r < v ? all[r].index : -1;
+    free(all);
+    return v;
+}
+
+/* ------------------------------------------------------------------ */
 /* Knob decoding and feature program (Sec. 2 "Configuration Explorer") */
 /* ------------------------------------------------------------------ */
 

@@ -73,6 +73,8 @@ def _load():
         lib.orc_topk.restype = i64
         lib.orc_screen.argtypes = [P, i64, i32, P, i32, i32, P, i32, i32, f32, i32, P, P, P]
         lib.orc_screen.restype = i64
+        lib.orc_rerank.argtypes = [P, i32, P, i64, P, i32, i32, i32, P, P]
+        lib.orc_rerank.restype = i64
         lib.orc_decode.argtypes = [P, i32, i64, i64, P]
         lib.orc_decode.restype = i32
         lib.orc_features.argtypes = [P, P, i32, P, i32, i64, i64, P, P]
@@ -214,6 +216,21 @@ def screen(feats, v_ens, p_ens, thr: float, k: int):
     if s < 0:
         raise ValueError("oracle screen failed (threshold outside (0,1) or no memory)")
     return pvalid, perf, out, int(s)
+
+
+def rerank(feats, cand, a_ens, n_final: int):
+    """Model A rerank of the kept candidates: (scores [m], final [n_final])."""
+    lib = _load()
+    an, at, ad = _ens(a_ens)
+    feats = _f32_2d(feats)
+    cand = np.ascontiguousarray(cand, dtype=np.int64)
+    score = np.empty(cand.size, np.float32)
+    final = np.empty(int(n_final), np.int64)
+    v = lib.orc_rerank(_ptr(feats), feats.shape[1], _ptr(cand), cand.size, _ptr(an), at, ad,
+                       int(n_final), _ptr(score), _ptr(final))
+    if v < 0:
+        raise MemoryError("oracle rerank allocation failed")
+    return score, final
 
 
 def decode(radices, first: int, n: int) -> np.ndarray:

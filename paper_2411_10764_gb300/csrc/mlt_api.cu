@@ -82,6 +82,7 @@ struct ScratchOwner {
   void* block = nullptr;  // one allocation for everything sized by n
   SelectState* state = nullptr;
   unsigned int* err = nullptr;
+  unsigned long long* rerank_keys = nullptr;  // [kMaxK]
   // host-buffer entry point staging
   long long host_cap_n = -1;
   int host_cap_F = 0;
@@ -156,6 +157,7 @@ int ensure_scratch(long long n) {
     MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(unsigned int)), "cudaMemset(error word)");
     MLT_CUDA(cudaMalloc(&g_scr.state, sizeof(SelectState)), "cudaMalloc(select state)");
     MLT_CUDA(cudaMemset(g_scr.state, 0, sizeof(SelectState)), "cudaMemset(select state)");
+    MLT_CUDA(cudaMalloc(&g_scr.rerank_keys, sizeof(unsigned long long) * kMaxK), "cudaMalloc(rerank keys)");
     g_scr.device = dev;
   }
   if (n > g_scr.cap_n) {
@@ -382,10 +384,11 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
         uint32_t meta;
         if (nd.feature >= 0) {
           const uint32_t left = static_cast<uint32_t>(order.size());
-          if (left > 0x3FFFu) return fail(MLT_EINVAL, "tree %d has too many nodes", t);
+          if (left > kCompactChildMask) return fail(MLT_EINVAL, "tree %d has too many nodes", t);
           order.push_back(2 * order[q] + 1);
           order.push_back(2 * order[q] + 2);
-          meta = static_cast<uint32_t>(nd.feature) | (left << 16) | (nd.default_left ? kMetaDefaultLeft : 0u);
+          meta = static_cast<uint32_t>(nd.feature) | (left << kCompactChildShift) |
+                 (nd.default_left ? kMetaDefaultLeft : 0u);
         } else {
           meta = kMetaLeaf;
         }
@@ -615,6 +618,31 @@ int mlt_screen_noalloc(void* stream, const float* feats, int64_t n, float thr, i
   return run_screen_with(st, feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk, s, false);
 }
 
+int mlt_rerank(void* stream, const float* feats, int64_t n, const int64_t* cand, int m, int n_final,
+               float* out_score, int64_t* out_final) {
+  if (n < 0 || n > 0x7FFFFFFFLL) return fail(MLT_EINVAL, "n must lie in [0, 2^31-1]");
+  if (m < 0 || m > kMaxK) return fail(MLT_EINVAL, "m must lie in [0, %d], got %d", kMaxK, m);
+  if (n_final < 1 || n_final > kMaxK) return fail(MLT_EINVAL, "n_final must lie in [1, %d], got %d", kMaxK, n_final);
+  if ((m > 0 && (cand == nullptr || out_score == nullptr || (n > 0 && feats == nullptr))) || out_final == nullptr)
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  const Model& A = g_models[MLT_MODEL_A];
+  if (!A.loaded) return fail(MLT_ENOMODEL, "model A is not loaded");
+  if (A.F != g_F) return fail(MLT_ENOMODEL, "model A was loaded for F=%d, current F=%d", A.F, g_F);
+  if (A.device != dev) return fail(MLT_EINVAL, "model A lives on device %d, current device is %d", A.device, dev);
+  rc = ensure_scratch(0);
+  if (rc != MLT_OK) return rc;
+  MLT_CUDA(launch_rerank(A.dm, feats, g_F, n, cand, m, n_final, out_score, out_final, g_scr.rerank_keys, g_scr.err,
+                         static_cast<cudaStream_t>(stream)),
+           "rerank launch");
+  g_launches += (m > 0 ? 1 : 0) + 1;
+  return MLT_OK;
+}
+
 int mlt_screen_decoded(void* stream, const int32_t* radices, const float* option_values, int n_knobs,
                        const mlt_feat_op* program, int64_t first_index, int64_t n, float thr, int k,
                        float* out_pvalid, float* out_perf, int64_t* out_topk) {
@@ -698,6 +726,7 @@ int mlt_sync_status(void* stream) {
   if (word == 0) return MLT_OK;
   MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(word)), "error word reset");
   if (word & kErrWaitTimeout) return fail(MLT_ETIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
+  if (word & kErrBadIndex) return fail(MLT_EINVAL, "a rerank candidate index was outside [0, n) (error word 0x%x)", word);
   return fail(MLT_ECUDA, "device-side bookkeeping error (error word 0x%x)", word);
 }
 

@@ -14,12 +14,13 @@ constexpr int kMaxOptions = 256;
 constexpr int kMaxProgram = 256;
 constexpr int kMaxF = 1024;
 constexpr int kMaxK = 16384;
-constexpr int kMaxDepth = 12;
+constexpr int kMaxDepth = 14;  // model A of the paper has depth 14 (Table 3)
 constexpr int kMaxFullDepth = 10;  // deeper ensembles use the compact table
 
 // Device error bits (accumulated in one word, read by mlt_sync_status).
 constexpr unsigned kErrWaitTimeout = 1u;  // an mbarrier wait gave up
 constexpr unsigned kErrSelect = 2u;       // top-k bookkeeping out of range
+constexpr unsigned kErrBadIndex = 4u;     // a rerank candidate index outside [0, n)
 
 // A bounded device wait gives up after this many nanoseconds.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
@@ -47,8 +48,8 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 // align16(4 * n_trees)), then each tree's existing nodes in breadth-first
 // order as {float value; uint32 meta}:
 //   meta bit 30 = leaf (value = leaf output), bit 31 = NaN goes left,
-//   bits 16..29 = index of the left child within the tree (right = left+1),
-//   bits 0..15 = feature index.
+//   bits 10..29 = index of the left child within the tree (right = left+1),
+//   bits 0..9 = feature index (F <= 1024).
 enum TableKind : int { kTableFull = 0, kTableCompact = 1 };
 
 struct FullLayout {
@@ -74,6 +75,9 @@ __host__ __device__ constexpr FullLayout full_layout(int D) {
 
 constexpr uint32_t kMetaLeaf = 1u << 30;
 constexpr uint32_t kMetaDefaultLeft = 1u << 31;
+constexpr uint32_t kCompactFeatureMask = 0x3FFu;  // bits 0..9
+constexpr uint32_t kCompactChildShift = 10;       // bits 10..29
+constexpr uint32_t kCompactChildMask = 0xFFFFFu;
 
 struct DeviceModel {
   const unsigned char* table = nullptr;
@@ -224,5 +228,11 @@ cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_
                            cudaStream_t st);
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base,
                         int64_t* out_topk, int sms, cudaStream_t st);
+
+// rerank.cu
+cudaError_t launch_rerank(const DeviceModel& A, const float* feats, int F, long long n,
+                          const int64_t* cand, int m, int n_final, float* out_score,
+                          int64_t* out_final, unsigned long long* keys, unsigned* err,
+                          cudaStream_t st);
 
 }  // namespace mlt

@@ -548,10 +548,10 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
           leaf[g] = __uint_as_float(r.x);
           live[g] = false;
         } else {
-          const float x = xs[(r.y & 0xFFFFu) * TC + tid];
+          const float x = xs[(r.y & kCompactFeatureMask) * TC + tid];
           uint32_t right = x >= __uint_as_float(r.x) ? 1u : 0u;
           if ((x != x) && !(r.y & kMetaDefaultLeft)) right = 1u;
-          j[g] = ((r.y >> 16) & 0x3FFFu) + right;
+          j[g] = ((r.y >> kCompactChildShift) & kCompactChildMask) + right;
         }
       }
     }

@@ -69,6 +69,7 @@ def lib(build_if_missing: bool = True):
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_shape": [i32, i32, i32, i32],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
+            "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
         }
         for name, args in sig.items():
             fn = getattr(L, name)
@@ -176,6 +177,23 @@ def screen_noalloc(feats, thr: float, k: int, out_pvalid=None, out_perf=None, ou
     _check(lib().mlt_screen_noalloc(_stream_ptr(stream), _dptr(feats), n, C.c_float(thr), int(k),
                                     _dptr(pv), _dptr(pf), _dptr(tk)))
     return pv, pf, tk
+
+
+def rerank(feats, cand, n_final: int, out_score=None, out_final=None, stream=None):
+    """Model A's rerank of candidate indices `cand` (CUDA int64 tensor) whose
+    rows are in `feats`: returns (scores [m], final [n_final])."""
+    import torch
+
+    if not (isinstance(cand, torch.Tensor) and cand.is_cuda and cand.dtype == torch.int64):
+        raise TypeError("cand must be an int64 CUDA tensor")
+    m = cand.numel()
+    if out_score is None:
+        out_score = torch.empty(m, dtype=torch.float32, device=cand.device)
+    if out_final is None:
+        out_final = torch.empty(int(n_final), dtype=torch.int64, device=cand.device)
+    _check(lib().mlt_rerank(_stream_ptr(stream), _dptr(feats), feats.shape[0], _dptr(cand), m, int(n_final),
+                            _dptr(out_score), _dptr(out_final)))
+    return out_score, out_final
 
 
 def screen_host(feats: np.ndarray, thr: float, k: int, out=None, stream=None):

@@ -232,20 +232,25 @@ class _RangeThresholds:
         return t.astype(np.float32)
 
 
-def make_ensemble(cfg: ScreenConfig, which: str, thresholds, seed: int) -> Ensemble:
-    """Random ensemble for model 'V' or 'P' in heap order."""
-    n_trees = cfg.v_trees if which == "V" else cfg.p_trees
-    depth = cfg.v_depth if which == "V" else cfg.p_depth
-    rng = _rng(seed, cfg.id, 2, 0 if which == "V" else 1)
+def make_ensemble(cfg: ScreenConfig, which: str, thresholds, seed: int, n_trees: int | None = None,
+                  depth: int | None = None, split_prob: float = 0.9, shape: str | None = None) -> Ensemble:
+    """Random ensemble for model 'V', 'P' or 'A' in heap order (n_trees,
+    depth and shape default to the workload's V / P settings)."""
+    if n_trees is None:
+        n_trees = cfg.v_trees if which == "V" else cfg.p_trees
+    if depth is None:
+        depth = cfg.v_depth if which == "V" else cfg.p_depth
+    shape = cfg.shape if shape is None else shape
+    rng = _rng(seed, cfg.id, 2, {"V": 0, "P": 1, "A": 2}[which])
     slots = (2 << depth) - 1
     nodes = np.zeros((n_trees, slots), dtype=NODE_DTYPE)
     slot_depth = np.floor(np.log2(np.arange(slots) + 1)).astype(np.int64)
-    if cfg.shape == "full":
+    if shape == "full":
         split = np.broadcast_to(slot_depth < depth, (n_trees, slots)).copy()
         leaf = ~split
     else:
         # unbalanced: the root always splits; a node at depth 1..depth-1 that
-        # exists splits with probability 0.9; nodes at `depth` are leaves
+        # exists splits with probability split_prob; nodes at `depth` are leaves
         split = np.zeros((n_trees, slots), dtype=bool)
         leaf = np.zeros((n_trees, slots), dtype=bool)
         exists = np.zeros((n_trees, slots), dtype=bool)
@@ -258,7 +263,7 @@ def make_ensemble(cfg: ScreenConfig, which: str, thresholds, seed: int) -> Ensem
             if d == 0:
                 s = exists[:, a:b]
             elif d < depth:
-                s = exists[:, a:b] & (rng.random(size=(n_trees, b - a)) < 0.9)
+                s = exists[:, a:b] & (rng.random(size=(n_trees, b - a)) < split_prob)
             else:
                 s = np.zeros((n_trees, b - a), dtype=bool)
             split[:, a:b] = s
@@ -415,6 +420,23 @@ def conv2d_decoder(seed: int, F: int = 96) -> Decoder:
     for i, (op, a, b, c) in enumerate(pg.ops[:F]):
         prog[i] = (op, a, b, c)
     return Decoder(radices, option_values, prog, pg.ranges[:F])
+
+
+def make_model_a(w: "Workload", seed: int = 1, n_trees: int = 300, depth: int = 14,
+                 split_prob: float = 0.75) -> Ensemble:
+    """Model A for a workload: a deeper performance regressor (300 rounds,
+    depth 14 in Table 3) over the same feature columns, unbalanced (a node
+    below the root splits with probability split_prob), leaves N(0, 0.1)."""
+    cfg = w.cfg
+    if w.feats is not None:
+        sample = w.feats[: min(w.n, THRESHOLD_SAMPLE_ROWS)]
+        if sample.shape[0] == 0:
+            sample = make_features(cfg, seed, THRESHOLD_SAMPLE_ROWS)
+        th = _QuantileThresholds(sample)
+    else:
+        th = _RangeThresholds(w.decoder.ranges)
+    return make_ensemble(cfg, "A", th, seed, n_trees=n_trees, depth=depth, split_prob=split_prob,
+                         shape="unbalanced")
 
 
 # --------------------------------------------------------------------------

@@ -82,8 +82,8 @@ def test_ensemble_validation_rejects(case):
     elif case == "model_id":
         model = 3
     elif case == "depth":
-        depth = 13
-        nodes = np.zeros((2 << 13) - 1, mlt.NODE_DTYPE)
+        depth = 15
+        nodes = np.zeros((2 << 15) - 1, mlt.NODE_DTYPE)
     elif case == "trees":
         n_trees = 0
         nodes = nodes[:0]

@@ -189,3 +189,69 @@ def _sampled_full_size(cid, n_sample=1500):
 @pytest.mark.parametrize("cid", [3, 4, 5])
 def test_full_size_sampled(cid):
     _sampled_full_size(cid)
+
+
+# --------------------------------------------------------------------------
+# Model A rerank of the kept candidates
+# --------------------------------------------------------------------------
+
+def _gpu_rerank(w, a, cand, n_final):
+    import torch
+
+    mlt.load_ensemble(mlt.MLT_MODEL_A, a.nodes, a.n_trees, a.depth)
+    x = torch.from_numpy(w.feats).cuda()
+    c = torch.as_tensor(np.asarray(cand, np.int64)).cuda()
+    sc, fin = mlt.rerank(x, c, n_final)
+    mlt.sync_status()
+    return sc.cpu().numpy(), fin.cpu().numpy()
+
+
+@pytest.mark.parametrize("cid,shape,depth", [(2, "unbalanced", 14), (3, "unbalanced", 12), (1, "full", 8)])
+def test_rerank_of_screened_topk_matches_oracle(cid, shape, depth):
+    import torch
+
+    w = W.make_workload(cid, seed=2, n=12000)
+    a = W.make_ensemble(w.cfg, "A", W._QuantileThresholds(w.feats[:4096]), 3, n_trees=150, depth=depth,
+                        split_prob=0.8, shape=shape)
+    mlt.load_workload_models(w)
+    _, _, tk = mlt.screen(torch.from_numpy(w.feats).cuda(), w.thr, w.k)
+    cand = tk.cpu().numpy()
+    n_final = w.k // 2  # (alpha + 1) N kept, N final, alpha = 1
+    sc, fin = _gpu_rerank(w, a, cand, n_final)
+    osc, ofin = O.rerank(w.feats, cand, a, n_final)
+    assert_same_bits(sc, osc, "A scores")
+    assert np.array_equal(fin, ofin)
+
+
+def test_rerank_edge_cases():
+    w = W.make_workload(1, seed=4, n=3000)
+    a = W.make_model_a(w, n_trees=40, depth=10)
+    mlt.load_workload_models(w)
+    cases = [
+        ([17], 1),
+        ([5, -1, 5, 2999, 0, -1], 8),  # padding, a duplicate, n_final past the valid entries
+        ([-1, -1], 3),
+        (list(range(0, 3000, 7)), 64),
+    ]
+    for cand, n_final in cases:
+        sc, fin = _gpu_rerank(w, a, cand, n_final)
+        osc, ofin = O.rerank(w.feats, np.asarray(cand, np.int64), a, n_final)
+        assert_same_bits(sc, osc, "A scores")
+        assert np.array_equal(fin, ofin)
+
+
+def test_rerank_reports_out_of_range_index():
+    import torch
+
+    w = W.make_workload(1, seed=4, n=100)
+    a = W.make_model_a(w, n_trees=10, depth=6)
+    mlt.load_workload_models(w)
+    mlt.load_ensemble(mlt.MLT_MODEL_A, a.nodes, a.n_trees, a.depth)
+    x = torch.from_numpy(w.feats).cuda()
+    c = torch.tensor([3, 100, 7], dtype=torch.int64, device="cuda")
+    sc, fin = mlt.rerank(x, c, 3)
+    with pytest.raises(mlt.MltError) as e:
+        mlt.sync_status()
+    assert e.value.code == -1
+    assert np.isneginf(sc.cpu().numpy()[1])
+    mlt.sync_status()  # the error was cleared

@@ -254,3 +254,32 @@ def test_conv2d_features_hand_worked():
         knobs, f = O.features(dec.radices, dec.option_values, dec.program, case["index"], 1)
         assert knobs[0].tolist() == case["digits"]
         assert same_float(f[0, :60], np.array(case["features_0_59"], np.float32)), case["index"]
+
+
+# --------------------------------------------------------------------------
+# Model A rerank
+# --------------------------------------------------------------------------
+
+def test_rerank_hand_worked():
+    g = golden("screen_small.json")
+    a = (slots_to_nodes(g["A"], O.NODE_DTYPE), len(g["A"]), g["A_depth"])
+    x = np.stack([floats(r) for r in g["rows"]])
+    for case in g["rerank_cases"]:
+        score, final = O.rerank(x, g["rerank_cand"], a, case["n_final"])
+        assert same_float(score, floats(g["rerank_score"]))
+        assert final.tolist() == case["final"]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_rerank_equals_sorted_margins(seed):
+    rng = np.random.default_rng(seed)
+    w = W.make_workload(1, seed=seed + 1, n=500)
+    cand = rng.choice(500, size=40, replace=False).astype(np.int64)
+    cand[rng.random(40) < 0.2] = -1
+    score, final = O.rerank(w.feats, cand, w.p, 25)
+    m = O.margins(w.p, w.feats)
+    valid = [int(c) for c in cand if c >= 0]
+    want = sorted(valid, key=lambda c: (-float(m[c]), c))[:25]
+    assert final.tolist() == want + [-1] * (25 - len(want))
+    for i, c in enumerate(cand):
+        assert same_float(score[i], m[c] if c >= 0 else np.float32(-np.inf))
