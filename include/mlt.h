@@ -169,6 +169,36 @@ int mlt_screen_noalloc(void *stream, const float *feats, int64_t n, float thr, i
 int mlt_screen_host(void *stream, const float *feats_host, int64_t n, float thr, int k,
                     float *pvalid_host, float *perf_host, int64_t *topk_host);
 
+/* Batched accumulation (Sec. 2: the explorer applies models P and V until
+ * it has accumulated (alpha+1)N configurations): candidates 0 .. n_total-1
+ * are screened in consecutive batches of `batch`; after each batch the
+ * device adds the batch's valid candidates to a running count, and once
+ * that count reaches `target` every later batch is skipped on the device
+ * (all batches are enqueued up front; no host round trip per batch).
+ * out_topk = the k best valid candidates over every batch screened, by the
+ * same order as mlt_screen -- identical to mlt_screen over the consumed
+ * prefix [0, consumed).
+ *   feats      device [n_total][F] fp32
+ *   batch >= 1 (at most 65536 batches);  target >= 1
+ *   out_pvalid, out_perf: device [n_total] fp32 or NULL; entries of the
+ *              consumed prefix are written, later ones are left untouched
+ *   out_topk   device [k] int64
+ *   out_stats  device int64[3] or NULL: {consumed candidates, valid
+ *              candidates kept, batches screened}
+ * Asynchronous on `stream`. */
+int mlt_screen_until(void *stream, const float *feats, int64_t n_total, int64_t batch,
+                     int64_t target, float thr, int k, float *out_pvalid, float *out_perf,
+                     int64_t *out_topk, int64_t *out_stats);
+
+/* mlt_screen_until over decoded candidates first_index .. first_index +
+ * n_total - 1 of a knob space (see mlt_decode_knobs); out_topk holds
+ * candidate indices. */
+int mlt_screen_until_decoded(void *stream, const int32_t *radices, const float *option_values,
+                             int n_knobs, const mlt_feat_op *program, int64_t first_index,
+                             int64_t n_total, int64_t batch, int64_t target, float thr, int k,
+                             float *out_pvalid, float *out_perf, int64_t *out_topk,
+                             int64_t *out_stats);
+
 /* Model A rerank (Sec. 2, "Hidden Feature Extractor & ML Model A"): from the
  * (alpha+1)N candidates kept by screening, model A -- a performance
  * regressor over visible and hidden features, typically deeper than P

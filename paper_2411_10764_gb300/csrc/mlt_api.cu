@@ -9,6 +9,7 @@
 //   compaction (select.cu) -> ascending survivor list
 //   P pass (traverse.cu)  -> P score per survivor + 64-bit rank keys
 //   radix select + sort (select.cu) -> top-k indices
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -83,6 +84,7 @@ struct ScratchOwner {
   SelectState* state = nullptr;
   unsigned int* err = nullptr;
   unsigned long long* rerank_keys = nullptr;  // [kMaxK]
+  StreamState* stream = nullptr;              // batched accumulation
   // host-buffer entry point staging
   long long host_cap_n = -1;
   int host_cap_F = 0;
@@ -158,6 +160,7 @@ int ensure_scratch(long long n) {
     MLT_CUDA(cudaMalloc(&g_scr.state, sizeof(SelectState)), "cudaMalloc(select state)");
     MLT_CUDA(cudaMemset(g_scr.state, 0, sizeof(SelectState)), "cudaMemset(select state)");
     MLT_CUDA(cudaMalloc(&g_scr.rerank_keys, sizeof(unsigned long long) * kMaxK), "cudaMalloc(rerank keys)");
+    MLT_CUDA(cudaMalloc(&g_scr.stream, sizeof(StreamState)), "cudaMalloc(stream state)");
     g_scr.device = dev;
   }
   if (n > g_scr.cap_n) {
@@ -466,7 +469,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   MLT_CUDA(dec ? launch_traverse_dec(V, av, *dec, sv, tiles_v, st) : launch_traverse(V, av, sv, tiles_v, st),
            "V pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[1], st), "cudaEventRecord");
-  MLT_CUDA(launch_compact(s, n, sv.threads, tiles_v, st), "compaction launch");
+  MLT_CUDA(launch_compact(s, n, sv.threads, tiles_v, nullptr, st), "compaction launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[2], st), "cudaEventRecord");
 
   TraverseArgs ap = a;
@@ -481,7 +484,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   MLT_CUDA(dec ? launch_traverse_dec(P, ap, *dec, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
            "P pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[3], st), "cudaEventRecord");
-  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, sm_count(), st), "top-k launch");
+  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, sm_count(), nullptr, st), "top-k launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
   g_launches += (tiles_v > 0 ? 1 : 0) + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
   return MLT_OK;
@@ -508,6 +511,109 @@ int noalloc_scratch(int dev, Scratch* out) {
   out->cand = reinterpret_cast<unsigned long long*>(b + kCand);
   out->state = reinterpret_cast<SelectState*>(b + kState);
   out->err = reinterpret_cast<unsigned int*>(b + kErr);
+  return MLT_OK;
+}
+
+// Batched accumulation (ML^2Tuner Sec. 2: the explorer applies P and V
+// until (alpha+1)N configurations have accumulated): batches of `batch`
+// candidates are all enqueued; after each, a one-thread kernel adds the
+// batch's survivors to the running count and raises a device flag once it
+// reaches `target`, which makes every later batch's kernels return at once.
+// One top-k then ranks all survivors kept.  The result equals screening the
+// consumed prefix of the candidates as a single batch.
+int run_stream(cudaStream_t st, const float* feats, const DecodeParams* dec0, long long n_total, long long batch,
+               long long target, float thr, int k, float* out_pvalid, float* out_perf, int64_t* out_topk,
+               int64_t* out_stats) {
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  rc = check_models(dev);
+  if (rc != MLT_OK) return rc;
+  rc = ensure_scratch(n_total);  // every kept survivor's key fits
+  if (rc != MLT_OK) return rc;
+  const Scratch& s = g_scr.s;
+  StreamState* ss = g_scr.stream;
+  const DeviceModel& V = g_models[MLT_MODEL_V].dm;
+  const DeviceModel& P = g_models[MLT_MODEL_P].dm;
+  const long long per = std::min(batch, std::max(1LL, n_total));
+  const ScreenShape sv = plan_for(V, g_F, per, g_shape[MLT_MODEL_V]);
+  const ScreenShape sp = plan_for(P, g_F, (per + 1) / 2, g_shape[MLT_MODEL_P]);
+  if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
+  MLT_CUDA(cudaMemsetAsync(s.state, 0, sizeof(SelectState), st), "reset selection state");
+  MLT_CUDA(cudaMemsetAsync(ss, 0, sizeof(StreamState), st), "reset stream state");
+  const unsigned tgt = static_cast<unsigned>(std::min<long long>(target, 0xFFFFFFFFLL));
+  TraverseArgs a{};
+  a.F = g_F;
+  a.state = s.state;
+  a.rows = s.rows;
+  a.tau = validity_cut(thr);
+  a.masks = s.masks;
+  a.tile_counts = s.tile_counts;
+  a.keys = s.keys;
+  a.hist = s.state->hist;
+  a.tile_offsets = s.tile_offsets;
+  a.state_rw = s.state;
+  a.err = s.err;
+  a.decode = dec0 != nullptr;
+  a.stream = ss;
+  long long launches = 0;
+  for (long long b0 = 0; b0 < n_total; b0 += batch) {
+    const long long nb = std::min(batch, n_total - b0);
+    TraverseArgs ab = a;
+    ab.n = nb;
+    ab.pos_base = b0;
+    ab.feats = feats ? feats + b0 * g_F : nullptr;
+    ab.vec4 = (ab.feats != nullptr && (reinterpret_cast<uintptr_t>(ab.feats) & 15u) == 0 && (g_F & 3) == 0) ? 1 : 0;
+    ab.out_pvalid = out_pvalid ? out_pvalid + b0 : nullptr;
+    ab.out_perf = out_perf ? out_perf + b0 : nullptr;
+    DecodeParams d;
+    if (dec0) {
+      d = *dec0;
+      d.first_index += b0;
+    }
+    TraverseArgs av = ab;
+    av.p_pass = 0;
+    av.table = V.table;
+    av.n_trees = V.n_trees;
+    av.tree_bytes = V.tree_bytes;
+    av.chunk_trees = sv.chunk_trees;
+    av.nbuf = sv.nbuf;
+    av.max_depth = V.depth;
+    const long long tiles_v = (nb + sv.threads - 1) / sv.threads;
+    MLT_CUDA(dec0 ? launch_traverse_dec(V, av, d, sv, tiles_v, st) : launch_traverse(V, av, sv, tiles_v, st),
+             "V pass launch");
+    MLT_CUDA(launch_compact(s, nb, sv.threads, tiles_v, ss, st), "compaction launch");
+    TraverseArgs ap = ab;
+    ap.p_pass = 1;
+    ap.table = P.table;
+    ap.n_trees = P.n_trees;
+    ap.tree_bytes = P.tree_bytes;
+    ap.chunk_trees = sp.chunk_trees;
+    ap.nbuf = sp.nbuf;
+    ap.max_depth = P.depth;
+    const long long tiles_p = (nb + sp.threads - 1) / sp.threads;
+    MLT_CUDA(dec0 ? launch_traverse_dec(P, ap, d, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
+             "P pass launch");
+    MLT_CUDA(launch_accumulate(ss, s.state, nb, tgt, st), "accumulate launch");
+    launches += 4;
+  }
+  MLT_CUDA(launch_topk(s, n_total, k, dec0 ? dec0->first_index : 0, out_topk, sm_count(), &ss->total, st),
+           "top-k launch");
+  launches += 1;
+  if (out_stats) {
+    MLT_CUDA(launch_stream_stats(ss, out_stats, st), "stats launch");
+    launches += 1;
+  }
+  g_launches += launches;
+  return MLT_OK;
+}
+
+int check_stream_args(long long n_total, long long batch, long long target, float thr, int k) {
+  int rc = check_screen_args(n_total, thr, k);
+  if (rc != MLT_OK) return rc;
+  if (batch < 1) return fail(MLT_EINVAL, "batch must be >= 1");
+  if (target < 1) return fail(MLT_EINVAL, "target must be >= 1");
+  if ((n_total + batch - 1) / batch > 65536) return fail(MLT_EINVAL, "more than 65536 batches");
   return MLT_OK;
 }
 
@@ -616,6 +722,33 @@ int mlt_screen_noalloc(void* stream, const float* feats, int64_t n, float thr, i
   // at zero (every other piece is rewritten before it is read)
   MLT_CUDA(cudaMemsetAsync(s.err, 0, sizeof(unsigned int), st), "clear static error word");
   return run_screen_with(st, feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk, s, false);
+}
+
+int mlt_screen_until(void* stream, const float* feats, int64_t n_total, int64_t batch, int64_t target, float thr,
+                     int k, float* out_pvalid, float* out_perf, int64_t* out_topk, int64_t* out_stats) {
+  int rc = check_stream_args(n_total, batch, target, thr, k);
+  if (rc != MLT_OK) return rc;
+  if ((n_total > 0 && feats == nullptr) || out_topk == nullptr) return fail(MLT_EINVAL, "feats and out_topk must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  return run_stream(static_cast<cudaStream_t>(stream), feats, nullptr, n_total, batch, target, thr, k, out_pvalid,
+                    out_perf, out_topk, out_stats);
+}
+
+int mlt_screen_until_decoded(void* stream, const int32_t* radices, const float* option_values, int n_knobs,
+                             const mlt_feat_op* program, int64_t first_index, int64_t n_total, int64_t batch,
+                             int64_t target, float thr, int k, float* out_pvalid, float* out_perf,
+                             int64_t* out_topk, int64_t* out_stats) {
+  int rc = check_stream_args(n_total, batch, target, thr, k);
+  if (rc != MLT_OK) return rc;
+  if (out_topk == nullptr) return fail(MLT_EINVAL, "out_topk must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  DecodeParams d;
+  rc = build_decoder(radices, option_values, n_knobs, program, g_F, first_index, n_total, &d);
+  if (rc != MLT_OK) return rc;
+  return run_stream(static_cast<cudaStream_t>(stream), nullptr, &d, n_total, batch, target, thr, k, out_pvalid,
+                    out_perf, out_topk, out_stats);
 }
 
 int mlt_rerank(void* stream, const float* feats, int64_t n, const int64_t* cand, int m, int n_final,

@@ -124,6 +124,17 @@ struct SelectState {
   unsigned int hist[kTopBins];  // 16-byte aligned
 };
 
+// Batched accumulation (mlt_screen_until): bookkeeping carried on the device
+// across the batches of one call.  Once `done` is set, every later batch's
+// kernels return at once (no host round trip decides when to stop).
+struct StreamState {
+  unsigned int total;           // survivors accumulated so far
+  unsigned int done;            // the target count was reached
+  unsigned int batches;         // batches screened
+  unsigned int pad;
+  unsigned long long consumed;  // candidates screened
+};
+
 struct Scratch {
   uint32_t* masks = nullptr;         // [ceil(n/32)] validity ballots
   uint32_t* tile_counts = nullptr;   // [n_tiles] survivors per V tile
@@ -166,6 +177,9 @@ struct TraverseArgs {
   unsigned int* hist;      // P pass: key histogram (kTopBins)
   unsigned int* err;
   int decode;              // features built from candidate indices
+  // batched accumulation (null: a single batch)
+  StreamState* stream;
+  long long pos_base;      // position of the batch's first candidate in the call
 };
 
 struct ScreenShape {
@@ -225,9 +239,13 @@ __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.lau
 
 // select.cu
 cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles,
-                           cudaStream_t st);
+                           const StreamState* ss, cudaStream_t st);
+// count: survivors to select from (null: the batch's own count)
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base,
-                        int64_t* out_topk, int sms, cudaStream_t st);
+                        int64_t* out_topk, int sms, const unsigned* count, cudaStream_t st);
+cudaError_t launch_accumulate(StreamState* ss, const SelectState* st_, long long n_batch,
+                              unsigned target, cudaStream_t st);
+cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaStream_t st);
 
 // rerank.cu
 cudaError_t launch_rerank(const DeviceModel& A, const float* feats, int F, long long n,

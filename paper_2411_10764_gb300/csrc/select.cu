@@ -24,10 +24,11 @@ constexpr int kTopkThreads = 512;
 constexpr int kSortMin = 8192;  // sort buffer entries (at least pow2(k))
 
 __global__ void __launch_bounds__(256)
-    k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n) {
+    k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n, const StreamState* ss) {
   __shared__ unsigned wc[32];
   pdl_wait();
   pdl_trigger();
+  if (ss && *reinterpret_cast<volatile const unsigned*>(&ss->done)) return;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const long long tile0 = static_cast<long long>(blockIdx.x) * blockDim.x;
   const long long first = tile0 + warp * 32;
@@ -61,14 +62,14 @@ __device__ void sort_desc(unsigned long long* sk, int n2) {
 
 __global__ void __launch_bounds__(kTopkThreads)
     k_topk(const unsigned long long* keys, unsigned long long* cand, SelectState* st, int k, int cap,
-           long long base, int64_t* out, unsigned* err) {
+           long long base, int64_t* out, unsigned* err, const unsigned* count) {
   extern __shared__ __align__(16) unsigned long long sk[];  // cap entries
   __shared__ unsigned warp_sum[kTopkThreads / 32];
   __shared__ unsigned s_bin, s_last, s_digit, s_rem, s_h, s_cnt;
   __shared__ unsigned h256[256];
   pdl_wait();
   const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const unsigned S = st->survivors;
+  const unsigned S = count ? *count : st->survivors;
   const unsigned kk = S < static_cast<unsigned>(k) ? S : static_cast<unsigned>(k);
 
   // 1. bucket of the kk-th largest key.  Thread t holds the 8 bins
@@ -201,17 +202,51 @@ __global__ void __launch_bounds__(kTopkThreads)
 
 }  // namespace
 
-cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, cudaStream_t st) {
+cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_tiles, const StreamState* ss,
+                           cudaStream_t st) {
   if (n_tiles <= 0) {
     // no V pass ran: start the selection state from zero survivors
     return cudaMemsetAsync(s.state, 0, sizeof(SelectState), st);
   }
   return launch_pdl(k_scatter, dim3(static_cast<unsigned>(n_tiles)), dim3(tile), 0, st, s.masks,
-                    static_cast<const uint32_t*>(s.tile_offsets), s.rows, n);
+                    static_cast<const uint32_t*>(s.tile_offsets), s.rows, n, ss);
+}
+
+namespace {
+
+// After a batch: add its survivors and candidates to the running counts and
+// raise `done` once the target is reached.
+__global__ void k_accumulate(StreamState* ss, const SelectState* st, long long n_batch, unsigned target) {
+  pdl_wait();
+  if (threadIdx.x != 0 || ss->done) return;
+  ss->total += st->survivors;
+  ss->consumed += static_cast<unsigned long long>(n_batch);
+  ss->batches += 1u;
+  if (ss->total >= target) ss->done = 1u;
+}
+
+__global__ void k_stream_stats(const StreamState* ss, int64_t* out) {
+  pdl_wait();
+  if (threadIdx.x == 0) {
+    out[0] = static_cast<int64_t>(ss->consumed);
+    out[1] = static_cast<int64_t>(ss->total);
+    out[2] = static_cast<int64_t>(ss->batches);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_accumulate(StreamState* ss, const SelectState* st_, long long n_batch, unsigned target,
+                              cudaStream_t st) {
+  return launch_pdl(k_accumulate, dim3(1), dim3(32), 0, st, ss, st_, n_batch, target);
+}
+
+cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaStream_t st) {
+  return launch_pdl(k_stream_stats, dim3(1), dim3(32), 0, st, ss, out_stats);
 }
 
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk, int sms,
-                        cudaStream_t st) {
+                        const unsigned* count, cudaStream_t st) {
   int cap = kSortMin;
   while (cap < k) cap <<= 1;
   const size_t smem = static_cast<size_t>(cap) * 8;
@@ -222,7 +257,7 @@ cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_ba
   if (g > 4LL * sms) g = 4LL * sms;
   return launch_pdl(k_topk, dim3(static_cast<unsigned>(g)), dim3(kTopkThreads), smem, st,
                     static_cast<const unsigned long long*>(s.keys), s.cand, s.state, k, cap, index_base, out_topk,
-                    s.err);
+                    s.err, count);
 }
 
 }  // namespace mlt

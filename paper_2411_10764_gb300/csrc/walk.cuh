@@ -211,7 +211,7 @@ __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodePar
 // Exclusive scan of the per-tile survivor counts by one CTA, then the
 // survivor total and a fresh selection state for the P pass and top-k.
 __device__ __forceinline__ void scan_tiles(const uint32_t* counts, uint32_t* offsets, long long n_tiles,
-                                           SelectState* st) {
+                                           SelectState* st, bool reset_hist) {
   __shared__ unsigned warp_sum[32];
   __shared__ unsigned carry;
   const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = T >> 5;
@@ -241,7 +241,8 @@ __device__ __forceinline__ void scan_tiles(const uint32_t* counts, uint32_t* off
     st->ticket = 0u;
     st->v_ticket = 0u;
   }
-  for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
+  if (reset_hist)
+    for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
   (void)nw;
 }
 __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_t* rowidx,
@@ -252,9 +253,12 @@ __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_
     unsigned bin = 0xFFFFFFFFu;
     if (in) {
       const uint32_t pos = rowidx[tid];
-      a.out_perf[pos] = acc;
-      const unsigned long long key = make_key(acc, pos);
-      a.keys[tile0 + tid] = key;
+      if (a.out_perf) a.out_perf[pos] = acc;
+      // batched accumulation: keys of all batches side by side, positions
+      // counted from the call's first candidate
+      const long long key_base = a.stream ? static_cast<long long>(a.stream->total) : 0;
+      const unsigned long long key = make_key(acc, static_cast<uint32_t>(a.pos_base + pos));
+      a.keys[key_base + tile0 + tid] = key;
       bin = static_cast<unsigned>(key >> (64 - kTopBits));
     }
     // one atomic per distinct bucket of the warp
@@ -266,8 +270,8 @@ __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_
   const long long i = tile0 + tid;
   const bool valid = in && (acc >= a.tau);
   if (in) {
-    a.out_pvalid[i] = sigmoid_f(acc);
-    if (!valid) a.out_perf[i] = -INFINITY;
+    if (a.out_pvalid) a.out_pvalid[i] = sigmoid_f(acc);
+    if (!valid && a.out_perf) a.out_perf[i] = -INFINITY;
   }
   const unsigned ball = __ballot_sync(0xFFFFFFFFu, valid);
   const int warp = tid >> 5;
@@ -289,7 +293,8 @@ __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_
     // the last V tile to finish turns the tile counts into offsets and
     // resets the selection state (no CTA waits for another)
     __threadfence();
-    scan_tiles(a.tile_counts, a.tile_offsets, gridDim.x, a.state_rw);
+    // batched accumulation keeps the key histogram of earlier batches
+    scan_tiles(a.tile_counts, a.tile_offsets, gridDim.x, a.state_rw, a.stream == nullptr);
   }
 }
 
@@ -423,8 +428,10 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   const int tid = threadIdx.x;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
   // the P pass needs the survivor count of the kernels before it; the V
-  // pass only needs them before it reads the features
-  if (a.p_pass) pdl_wait();
+  // pass only needs them before it reads the features, unless a batched call
+  // must first learn whether an earlier batch already reached its target
+  if (a.p_pass || a.stream) pdl_wait();
+  if (a.stream && *reinterpret_cast<volatile const unsigned*>(&a.stream->done)) return;
   const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
   if (tile0 >= count) return;  // whole CTA, before any copy is issued
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
@@ -513,6 +520,7 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
   const int tid = threadIdx.x;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
   pdl_wait();
+  if (a.stream && *reinterpret_cast<volatile const unsigned*>(&a.stream->done)) return;
   const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
   if (tile0 >= count) return;
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));

@@ -70,6 +70,8 @@ def lib(build_if_missing: bool = True):
             "mlt_tune_shape": [i32, i32, i32, i32],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
+            "mlt_screen_until": [P, P, i64, i64, i64, f32, i32, P, P, P, P],
+            "mlt_screen_until_decoded": [P, P, P, i32, P, i64, i64, i64, i64, f32, i32, P, P, P, P],
         }
         for name, args in sig.items():
             fn = getattr(L, name)
@@ -177,6 +179,38 @@ def screen_noalloc(feats, thr: float, k: int, out_pvalid=None, out_perf=None, ou
     _check(lib().mlt_screen_noalloc(_stream_ptr(stream), _dptr(feats), n, C.c_float(thr), int(k),
                                     _dptr(pv), _dptr(pf), _dptr(tk)))
     return pv, pf, tk
+
+
+def screen_until(feats, batch: int, target: int, thr: float, k: int, with_outputs=True, stream=None):
+    """Batched accumulation over the rows of `feats`: returns (pvalid, perf,
+    topk, stats) with stats = [consumed, kept, batches] (CUDA tensors)."""
+    import torch
+
+    n = feats.shape[0]
+    pv = torch.empty(n, dtype=torch.float32, device=feats.device) if with_outputs else None
+    pf = torch.empty(n, dtype=torch.float32, device=feats.device) if with_outputs else None
+    tk = torch.empty(int(k), dtype=torch.int64, device=feats.device)
+    stats = torch.empty(3, dtype=torch.int64, device=feats.device)
+    _check(lib().mlt_screen_until(_stream_ptr(stream), _dptr(feats), n, int(batch), int(target), C.c_float(thr),
+                                  int(k), _dptr(pv), _dptr(pf), _dptr(tk), _dptr(stats)))
+    return pv, pf, tk, stats
+
+
+def screen_until_decoded(radices, option_values, program, first_index: int, n_total: int, batch: int,
+                         target: int, thr: float, k: int, device="cuda", with_outputs=True, stream=None):
+    """Batched accumulation over a decoded knob space."""
+    import torch
+
+    r, ov, prog = _decoder_args(radices, option_values, program)
+    pv = torch.empty(n_total, dtype=torch.float32, device=device) if with_outputs else None
+    pf = torch.empty(n_total, dtype=torch.float32, device=device) if with_outputs else None
+    tk = torch.empty(int(k), dtype=torch.int64, device=device)
+    stats = torch.empty(3, dtype=torch.int64, device=device)
+    _check(lib().mlt_screen_until_decoded(_stream_ptr(stream), r.ctypes.data, ov.ctypes.data, r.size,
+                                          prog.ctypes.data, int(first_index), int(n_total), int(batch),
+                                          int(target), C.c_float(thr), int(k), _dptr(pv), _dptr(pf),
+                                          _dptr(tk), _dptr(stats)))
+    return pv, pf, tk, stats
 
 
 def rerank(feats, cand, n_final: int, out_score=None, out_final=None, stream=None):

@@ -255,3 +255,70 @@ def test_rerank_reports_out_of_range_index():
     assert e.value.code == -1
     assert np.isneginf(sc.cpu().numpy()[1])
     mlt.sync_status()  # the error was cleared
+
+
+# --------------------------------------------------------------------------
+# Batched accumulation: screen batch after batch until enough survivors
+# --------------------------------------------------------------------------
+
+def _expected_prefix(valid, n, batch, target):
+    """(consumed, kept, batches) of the accumulation rule on oracle decisions."""
+    kept = 0
+    for b, b0 in enumerate(range(0, n, batch)):
+        b1 = min(n, b0 + batch)
+        kept += int(valid[b0:b1].sum())
+        if kept >= target:
+            return b1, kept, b + 1
+    return n, kept, -(-n // batch)
+
+
+@pytest.mark.parametrize("target,batch", [(1, 4096), (3000, 4096), (9000, 3000), (10 ** 9, 4096), (5000, 20000)])
+def test_screen_until_equals_oracle_on_the_consumed_prefix(target, batch):
+    import torch
+
+    w = W.make_workload(2, seed=3, n=20000)
+    mlt.load_workload_models(w)
+    pv, pf, tk, stats = mlt.screen_until(torch.from_numpy(w.feats).cuda(), batch, target, w.thr, w.k)
+    mlt.sync_status()
+    opv, opf, valid, _ = O.screen_rows(w.feats, w.v, w.p, w.thr, threads=THREADS)
+    consumed, kept, batches = _expected_prefix(valid, w.n, batch, target)
+    assert stats.cpu().tolist() == [consumed, kept, batches]
+    want, _ = O.topk(opf[:consumed], valid[:consumed], w.k)
+    assert np.array_equal(tk.cpu().numpy(), want)
+    assert_same_bits(pf.cpu().numpy()[:consumed], opf[:consumed], "perf (consumed prefix)")
+    assert_pvalid(pv.cpu().numpy()[:consumed], opv[:consumed])
+
+
+def test_screen_until_decoded_space():
+    w = W.make_workload(4, seed=1, n=30000)
+    d = w.decoder
+    first, batch, target = 777777, 8192, 6000
+    mlt.load_workload_models(w)
+    pv, pf, tk, stats = mlt.screen_until_decoded(d.radices, d.option_values, d.program, first, w.n, batch,
+                                                 target, w.thr, w.k)
+    mlt.sync_status()
+    _, x = O.features(d.radices, d.option_values, d.program, first, w.n, threads=THREADS)
+    opv, opf, valid, _ = O.screen_rows(x, w.v, w.p, w.thr, threads=THREADS)
+    consumed, kept, batches = _expected_prefix(valid, w.n, batch, target)
+    assert stats.cpu().tolist() == [consumed, kept, batches]
+    want, _ = O.topk(opf[:consumed], valid[:consumed], w.k, index_base=first)
+    assert np.array_equal(tk.cpu().numpy(), want)
+    assert_same_bits(pf.cpu().numpy()[:consumed], opf[:consumed], "perf (consumed prefix)")
+
+
+def test_screen_until_without_per_candidate_outputs_and_repeat():
+    import torch
+
+    w = W.make_workload(1, seed=6, n=10000)
+    mlt.load_workload_models(w)
+    x = torch.from_numpy(w.feats).cuda()
+    first = mlt.screen_until(x, 1000, 2500, w.thr, w.k, with_outputs=False)
+    second = mlt.screen_until(x, 1000, 2500, w.thr, w.k, with_outputs=False)
+    mlt.sync_status()
+    assert np.array_equal(first[2].cpu().numpy(), second[2].cpu().numpy())
+    assert first[3].cpu().tolist() == second[3].cpu().tolist()
+    _, opf, valid, _ = O.screen_rows(w.feats, w.v, w.p, w.thr)
+    consumed, kept, batches = _expected_prefix(valid, w.n, 1000, 2500)
+    assert first[3].cpu().tolist() == [consumed, kept, batches]
+    want, _ = O.topk(opf[:consumed], valid[:consumed], w.k)
+    assert np.array_equal(first[2].cpu().numpy(), want)
