@@ -122,7 +122,7 @@ ScreenShape plan_compact(int F, long long n_eff, int sms, int optin, const Shape
       best.smem = smem;
     }
   }
-  best.group = 4;
+  best.group = 8;
   return best;
 }
 
@@ -141,10 +141,10 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     e = launch_pdl(k, grid, block, shape.smem, st, args);
     if (e != cudaSuccess) return e;
   } else {
-    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_traverse_compact<4>, grid, block, shape.smem, st, args);
+    e = launch_pdl(k_traverse_compact<8>, grid, block, shape.smem, st, args);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

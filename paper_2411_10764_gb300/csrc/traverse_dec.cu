@@ -78,11 +78,11 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     e = launch_pdl(k, grid, block, shape.smem, st, args, dec);
     if (e != cudaSuccess) return e;
   } else {
-    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact_dec<4>,
+    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact_dec<8>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_traverse_compact_dec<4>, grid, block, shape.smem, st, args, dec);
+    e = launch_pdl(k_traverse_compact_dec<8>, grid, block, shape.smem, st, args, dec);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

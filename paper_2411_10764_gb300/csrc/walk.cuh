@@ -77,6 +77,32 @@ __device__ __forceinline__ unsigned long long global_ns() {
   return t;
 }
 
+// L2 cache policies for loads: node tables of the deep-tree walk are
+// re-read by every tile and should stay in L2 (evict_last); feature rows are
+// read once and should leave first (evict_first).
+__device__ __forceinline__ unsigned long long policy_evict_last() {
+  unsigned long long p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ unsigned long long policy_evict_first() {
+  unsigned long long p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint2 ldg_u2_hint(const uint2* ptr, unsigned long long pol) {
+  uint2 v;
+  asm("ld.global.nc.L2::cache_hint.v2.u32 {%0, %1}, [%2], %3;" : "=r"(v.x), "=r"(v.y) : "l"(ptr), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ float4 ldg_f4_hint(const float4* ptr, unsigned long long pol) {
+  float4 v;
+  asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+      : "l"(ptr), "l"(pol));
+  return v;
+}
+
 // Wait for an mbarrier phase, giving up after kWaitLimitNs.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -162,7 +188,7 @@ __device__ __forceinline__ bool decode_column(const DecodeParams& d, long long i
 // store hit 32 different banks).  Returns whether the row holds a NaN.
 __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodeParams* dec, float* xs,
                                           const uint32_t* rowidx, long long tile0, int rows_here,
-                                          int TC) {
+                                          int TC, bool read_once = false) {
   const int F = a.F;
   const int c = threadIdx.x;
   if (c >= rows_here) {
@@ -181,7 +207,7 @@ __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodePar
       float4 v[U];
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (q0 + u < F4) v[u] = __ldg(s4 + q0 + u);
+        if (q0 + u < F4) v[u] = read_once ? ldg_f4_hint(s4 + q0 + u, policy_evict_first()) : __ldg(s4 + q0 + u);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         if (q0 + u < F4) {
@@ -528,11 +554,13 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
   float* xs = reinterpret_cast<float*>(smem);
   uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + align_up(static_cast<size_t>(a.F) * TC * 4, 128));
   if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
-  __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+  // feature rows are read once; the node tables are re-read by every tile
+  __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC, true));
 
   const uint32_t* offs = reinterpret_cast<const uint32_t*>(a.table);
   const uint2* recs =
       reinterpret_cast<const uint2*>(a.table + align_up(static_cast<size_t>(a.n_trees) * 4, 16));
+  const unsigned long long keep = policy_evict_last();
   float acc = 0.0f;
   const int steps = a.max_depth + 1;
   for (int t = 0; t < a.n_trees; t += G) {
@@ -548,20 +576,27 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
       leaf[g] = 0.0f;
     }
     for (int s = 0; s < steps; ++s) {
+      // all G node loads first (a finished walk re-reads its leaf: the
+      // address stays inside its tree), then the decisions
+      uint2 r[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) r[g] = ldg_u2_hint(tr[g] + j[g], keep);
+      bool any = false;
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         if (!live[g]) continue;
-        const uint2 r = __ldg(tr[g] + j[g]);
-        if (r.y & kMetaLeaf) {
-          leaf[g] = __uint_as_float(r.x);
+        if (r[g].y & kMetaLeaf) {
+          leaf[g] = __uint_as_float(r[g].x);
           live[g] = false;
         } else {
-          const float x = xs[(r.y & kCompactFeatureMask) * TC + tid];
-          uint32_t right = x >= __uint_as_float(r.x) ? 1u : 0u;
-          if ((x != x) && !(r.y & kMetaDefaultLeft)) right = 1u;
-          j[g] = ((r.y >> kCompactChildShift) & kCompactChildMask) + right;
+          const float x = xs[(r[g].y & kCompactFeatureMask) * TC + tid];
+          uint32_t right = x >= __uint_as_float(r[g].x) ? 1u : 0u;
+          if ((x != x) && !(r[g].y & kMetaDefaultLeft)) right = 1u;
+          j[g] = ((r[g].y >> kCompactChildShift) & kCompactChildMask) + right;
+          any = true;
         }
       }
+      if (!__any_sync(0xFFFFFFFFu, any)) break;  // every walk of the warp is at a leaf
     }
 #pragma unroll
     for (int g = 0; g < G; ++g)
