@@ -199,6 +199,31 @@ int mlt_screen_until_decoded(void *stream, const int32_t *radices, const float *
                              float *out_pvalid, float *out_perf, int64_t *out_topk,
                              int64_t *out_stats);
 
+/* Explorer proposal step (Sec. 2, "Configuration Explorer": the explorer
+ * searches the knob space for configurations the models rank highest; the
+ * paper leaves the search open, and this call is one simulated-annealing
+ * move of m independent chains, TVM-style).  For chain i:
+ *   parent[i] < 0 or >= the size of the space: inactive (next = parent,
+ *     score copied, not accepted; an index past the space is also reported
+ *     by mlt_sync_status as MLT_EINVAL);
+ *   otherwise knob j = knob_draw[i] mod n_knobs of the parent is set to
+ *     option index digit_draw[i] mod r_j, giving proposal q;
+ *   q is screened like any candidate: s = margin_P(q) if valid, else -inf;
+ *   accepted iff s > -inf and fl(s - parent_score[i]) >= fl(temperature *
+ *     log_u[i]) (Metropolis: log_u[i] = ln of a uniform draw);
+ *   out_next[i] = accepted ? q : parent[i];
+ *   out_next_score[i] = accepted ? s : parent_score[i].
+ * The random words knob_draw, digit_draw and log_u are the caller's
+ * (device [m] uint32, uint32, fp32), so results are reproducible.
+ * Decoder arguments as for mlt_decode_knobs (program length = F); models V
+ * and P must be loaded.  parent, parent_score, outputs: device [m].
+ * temperature > 0; thr in (0, 1).  Asynchronous on `stream`. */
+int mlt_sa_step(void *stream, const int32_t *radices, const float *option_values, int n_knobs,
+                const mlt_feat_op *program, const int64_t *parent, const float *parent_score,
+                const uint32_t *knob_draw, const uint32_t *digit_draw, const float *log_u,
+                int64_t m, float temperature, float thr, int64_t *out_next,
+                float *out_next_score, int32_t *out_accepted);
+
 /* Model A rerank (Sec. 2, "Hidden Feature Extractor & ML Model A"): from the
  * (alpha+1)N candidates kept by screening, model A -- a performance
  * regressor over visible and hidden features, typically deeper than P

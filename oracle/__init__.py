@@ -12,6 +12,7 @@ from .oracle import (  # noqa: F401
     features,
     margins,
     rerank,
+    sa_step,
     screen,
     screen_rows,
     sigmoid,

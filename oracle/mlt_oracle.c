@@ -414,3 +414,75 @@ int orc_features(const int32_t *radices, const float *option_values,
     }
     return 0;
 }
+
+/* ------------------------------------------------------------------ */
+/* Explorer proposal step (Sec. 2 "Configuration Explorer")           */
+/* ------------------------------------------------------------------ */
+
+/* One simulated-annealing step over m chains of the knob space.  The paper
+ * leaves the explorer's search unspecified beyond "selects configurations
+ * with the highest potential"; this step is the build's reading:
+ *   chain i with parent[i] < 0 is inactive (next = parent, score copied);
+ *   otherwise knob j = knob_draw[i] mod n_knobs of the parent is set to
+ *   digit d = digit_draw[i] mod r_j, giving proposal q;
+ *   q is scored like any candidate: s = margin_P(q) if V finds it valid
+ *   (sigmoid(margin_V) >= thr), else -inf;
+ *   accept iff s > -inf and fl(s - parent_score[i]) >= fl(temperature *
+ *   log_u[i])  (Metropolis with the log of a uniform draw passed in);
+ *   next = accept ? q : parent, next_score = accept ? s : parent_score.
+ * Returns 0, or -1 on a malformed program / threshold. */
+int orc_sa_step(const int32_t *radices, const float *option_values, int n_knobs,
+                const orc_feat_op *program, int F, const orc_node *v_nodes, int v_trees,
+                int v_depth, const orc_node *p_nodes, int p_trees, int p_depth,
+                const int64_t *parent, const float *parent_score, const uint32_t *knob_draw,
+                const uint32_t *digit_draw, const float *log_u, int64_t m, float temperature,
+                float thr, int64_t *out_next, float *out_next_score, int32_t *out_accepted)
+{
+    float tau = orc_tau(thr);
+    if (isnan(tau) || n_knobs <= 0 || n_knobs > 64)
+        return -1;
+    float *row = (float *)malloc((size_t)(F > 0 ? F : 1) * sizeof(float));
+    if (!row)
+        return -1;
+    int rc = 0;
+    for (int64_t i = 0; i < m && rc == 0; ++i) {
+        if (parent[i] < 0) {
+            out_next[i] = parent[i];
+            out_next_score[i] = parent_score[i];
+            out_accepted[i] = 0;
+            continue;
+        }
+        /* parent's digits, knob 0 least significant */
+        int32_t digit[64];
+        int64_t rem = parent[i];
+        for (int j = 0; j < n_knobs; ++j) {
+            digit[j] = (int32_t)(rem % radices[j]);
+            rem /= radices[j];
+        }
+        int kj = (int)(knob_draw[i] % (uint32_t)n_knobs);
+        digit[kj] = (int32_t)(digit_draw[i] % (uint32_t)radices[kj]);
+        int64_t q = 0, place = 1;
+        for (int j = 0; j < n_knobs; ++j) {
+            q += digit[j] * place;
+            place *= radices[j];
+        }
+        uint8_t knobs[64];
+        if (orc_features(radices, option_values, n_knobs, program, F, q, 1, knobs, row) != 0) {
+            rc = -1;
+            break;
+        }
+        float mv = orc_margin(v_nodes, v_trees, v_depth, row);
+        float s = mv >= tau ? orc_margin(p_nodes, p_trees, p_depth, row) : -INFINITY;
+        int accept = 0;
+        if (s != -INFINITY) {
+            float d = s - parent_score[i];
+            float bar = temperature * log_u[i];
+            accept = d >= bar;
+        }
+        out_next[i] = accept ? q : parent[i];
+        out_next_score[i] = accept ? s : parent_score[i];
+        out_accepted[i] = accept;
+    }
+    free(row);
+    return rc;
+}

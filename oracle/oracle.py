@@ -75,6 +75,9 @@ def _load():
         lib.orc_screen.restype = i64
         lib.orc_rerank.argtypes = [P, i32, P, i64, P, i32, i32, i32, P, P]
         lib.orc_rerank.restype = i64
+        lib.orc_sa_step.argtypes = [P, P, i32, P, i32, P, i32, i32, P, i32, i32, P, P, P, P, P, i64, f32, f32,
+                                    P, P, P]
+        lib.orc_sa_step.restype = i32
         lib.orc_decode.argtypes = [P, i32, i64, i64, P]
         lib.orc_decode.restype = i32
         lib.orc_features.argtypes = [P, P, i32, P, i32, i64, i64, P, P]
@@ -231,6 +234,32 @@ def rerank(feats, cand, a_ens, n_final: int):
     if v < 0:
         raise MemoryError("oracle rerank allocation failed")
     return score, final
+
+
+def sa_step(radices, option_values, program, v_ens, p_ens, parent, parent_score, knob_draw, digit_draw,
+            log_u, temperature: float, thr: float):
+    """One explorer proposal step: (next [m] int64, next_score [m] f32, accepted [m] i32)."""
+    lib = _load()
+    r = np.ascontiguousarray(radices, dtype=np.int32)
+    ov = np.ascontiguousarray(option_values, dtype=np.float32)
+    prog = np.ascontiguousarray(program)
+    vn, vt, vd = _ens(v_ens)
+    pn, pt, pd = _ens(p_ens)
+    parent = np.ascontiguousarray(parent, dtype=np.int64)
+    ps = np.ascontiguousarray(parent_score, dtype=np.float32)
+    kd = np.ascontiguousarray(knob_draw, dtype=np.uint32)
+    dd = np.ascontiguousarray(digit_draw, dtype=np.uint32)
+    lu = np.ascontiguousarray(log_u, dtype=np.float32)
+    m = parent.size
+    nxt = np.empty(m, np.int64)
+    nsc = np.empty(m, np.float32)
+    acc = np.empty(m, np.int32)
+    rc = lib.orc_sa_step(_ptr(r), _ptr(ov), r.size, _ptr(prog), prog.size, _ptr(vn), vt, vd, _ptr(pn), pt, pd,
+                         _ptr(parent), _ptr(ps), _ptr(kd), _ptr(dd), _ptr(lu), m, float(temperature), float(thr),
+                         _ptr(nxt), _ptr(nsc), _ptr(acc))
+    if rc != 0:
+        raise ValueError("malformed program or threshold")
+    return nxt, nsc, acc
 
 
 def decode(radices, first: int, n: int) -> np.ndarray:

@@ -85,6 +85,12 @@ struct ScratchOwner {
   unsigned int* err = nullptr;
   unsigned long long* rerank_keys = nullptr;  // [kMaxK]
   StreamState* stream = nullptr;              // batched accumulation
+  // explorer proposal step buffers, grown with m
+  long long sa_cap = -1;
+  long long* sa_prop = nullptr;
+  float* sa_pvalid = nullptr;
+  float* sa_perf = nullptr;
+  int64_t* sa_topk = nullptr;
   // host-buffer entry point staging
   long long host_cap_n = -1;
   int host_cap_F = 0;
@@ -749,6 +755,59 @@ int mlt_screen_until_decoded(void* stream, const int32_t* radices, const float* 
   if (rc != MLT_OK) return rc;
   return run_stream(static_cast<cudaStream_t>(stream), nullptr, &d, n_total, batch, target, thr, k, out_pvalid,
                     out_perf, out_topk, out_stats);
+}
+
+int mlt_sa_step(void* stream, const int32_t* radices, const float* option_values, int n_knobs,
+                const mlt_feat_op* program, const int64_t* parent, const float* parent_score,
+                const uint32_t* knob_draw, const uint32_t* digit_draw, const float* log_u, int64_t m,
+                float temperature, float thr, int64_t* out_next, float* out_next_score, int32_t* out_accepted) {
+  if (m < 0 || m > 0x7FFFFFFFLL) return fail(MLT_EINVAL, "m must lie in [0, 2^31-1]");
+  if (!(thr > 0.0f && thr < 1.0f)) return fail(MLT_EINVAL, "thr must lie in (0, 1)");
+  if (!(temperature > 0.0f) || !std::isfinite(temperature)) return fail(MLT_EINVAL, "temperature must be positive");
+  if (m > 0 && (parent == nullptr || parent_score == nullptr || knob_draw == nullptr || digit_draw == nullptr ||
+                log_u == nullptr || out_next == nullptr || out_next_score == nullptr || out_accepted == nullptr))
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  DecodeParams d;
+  int rc = build_decoder(radices, option_values, n_knobs, program, g_F, 0, 0, &d);
+  if (rc != MLT_OK) return rc;
+  long double space_ld = 1.0L;
+  for (int j = 0; j < n_knobs; ++j) space_ld *= radices[j];
+  const long long space = space_ld > 9.0e18L ? static_cast<long long>(9.0e18L) : static_cast<long long>(space_ld);
+  if (m == 0) return MLT_OK;
+  rc = ensure_scratch(m);
+  if (rc != MLT_OK) return rc;
+  ScratchOwner& S = g_scr;
+  if (m > S.sa_cap) {
+    cudaDeviceSynchronize();
+    cudaFree(S.sa_prop);
+    cudaFree(S.sa_pvalid);
+    cudaFree(S.sa_perf);
+    cudaFree(S.sa_topk);
+    S.sa_prop = nullptr;
+    S.sa_pvalid = S.sa_perf = nullptr;
+    S.sa_topk = nullptr;
+    S.sa_cap = -1;
+    if (cudaMalloc(&S.sa_prop, sizeof(long long) * m) != cudaSuccess ||
+        cudaMalloc(&S.sa_pvalid, sizeof(float) * m) != cudaSuccess ||
+        cudaMalloc(&S.sa_perf, sizeof(float) * m) != cudaSuccess ||
+        cudaMalloc(&S.sa_topk, sizeof(int64_t)) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(MLT_ENOMEM, "cannot allocate proposal buffers");
+    }
+    S.sa_cap = m;
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  MLT_CUDA(launch_sa_propose(d, space, parent, knob_draw, digit_draw, m, S.sa_prop, S.err, st), "propose launch");
+  d.index_list = S.sa_prop;
+  rc = run_screen_with(st, nullptr, &d, m, thr, 1, S.sa_pvalid, S.sa_perf, S.sa_topk, g_scr.s, true);
+  if (rc != MLT_OK) return rc;
+  MLT_CUDA(launch_sa_accept(space, parent, parent_score, S.sa_prop, S.sa_perf, log_u, m, temperature, out_next,
+                            out_next_score, out_accepted, st),
+           "accept launch");
+  g_launches += 2;
+  return MLT_OK;
 }
 
 int mlt_rerank(void* stream, const float* feats, int64_t n, const int64_t* cand, int m, int n_final,

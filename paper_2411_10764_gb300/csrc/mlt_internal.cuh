@@ -95,6 +95,7 @@ struct DecodeParams {
   int n_knobs;
   int F;
   long long first_index;
+  const long long* index_list;  // device: candidate of position i (null: first_index + i)
   int radix[kMaxKnobs];
   int opt_off[kMaxKnobs];
   float opts[kMaxOptions];
@@ -246,6 +247,15 @@ cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_ba
 cudaError_t launch_accumulate(StreamState* ss, const SelectState* st_, long long n_batch,
                               unsigned target, cudaStream_t st);
 cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaStream_t st);
+
+// sa.cu (explorer proposal step)
+cudaError_t launch_sa_propose(const DecodeParams& dec, long long space, const int64_t* parent,
+                              const uint32_t* knob_draw, const uint32_t* digit_draw, long long m,
+                              long long* prop, unsigned* err, cudaStream_t st);
+cudaError_t launch_sa_accept(long long space, const int64_t* parent, const float* parent_score,
+                             const long long* prop, const float* perf, const float* log_u, long long m,
+                             float temperature, int64_t* out_next, float* out_next_score,
+                             int32_t* out_accepted, cudaStream_t st);
 
 // rerank.cu
 cudaError_t launch_rerank(const DeviceModel& A, const float* feats, int F, long long n,

@@ -196,7 +196,8 @@ __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodePar
     return false;
   }
   const long long pos = a.p_pass ? static_cast<long long>(rowidx[c]) : tile0 + c;
-  if (dec != nullptr) return decode_column(*dec, dec->first_index + pos, xs, TC, c);
+  if (dec != nullptr)
+    return decode_column(*dec, dec->index_list ? dec->index_list[pos] : dec->first_index + pos, xs, TC, c);
   bool nan = false;
   const float* src = a.feats + pos * F;
   if (a.vec4) {

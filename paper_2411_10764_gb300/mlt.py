@@ -72,6 +72,7 @@ def lib(build_if_missing: bool = True):
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
             "mlt_screen_until": [P, P, i64, i64, i64, f32, i32, P, P, P, P],
             "mlt_screen_until_decoded": [P, P, P, i32, P, i64, i64, i64, i64, f32, i32, P, P, P, P],
+            "mlt_sa_step": [P, P, P, i32, P, P, P, P, P, P, i64, f32, f32, P, P, P],
         }
         for name, args in sig.items():
             fn = getattr(L, name)
@@ -211,6 +212,24 @@ def screen_until_decoded(radices, option_values, program, first_index: int, n_to
                                           int(target), C.c_float(thr), int(k), _dptr(pv), _dptr(pf),
                                           _dptr(tk), _dptr(stats)))
     return pv, pf, tk, stats
+
+
+def sa_step(radices, option_values, program, parent, parent_score, knob_draw, digit_draw, log_u,
+            temperature: float, thr: float, stream=None):
+    """One explorer proposal step over the chains in `parent` (CUDA tensors:
+    int64, float32, uint32-as-int32, int32, float32): returns (next,
+    next_score, accepted) CUDA tensors."""
+    import torch
+
+    r, ov, prog = _decoder_args(radices, option_values, program)
+    m = parent.numel()
+    nxt = torch.empty(m, dtype=torch.int64, device=parent.device)
+    nsc = torch.empty(m, dtype=torch.float32, device=parent.device)
+    acc = torch.empty(m, dtype=torch.int32, device=parent.device)
+    _check(lib().mlt_sa_step(_stream_ptr(stream), r.ctypes.data, ov.ctypes.data, r.size, prog.ctypes.data,
+                             _dptr(parent), _dptr(parent_score), _dptr(knob_draw), _dptr(digit_draw), _dptr(log_u),
+                             m, C.c_float(temperature), C.c_float(thr), _dptr(nxt), _dptr(nsc), _dptr(acc)))
+    return nxt, nsc, acc
 
 
 def rerank(feats, cand, n_final: int, out_score=None, out_final=None, stream=None):

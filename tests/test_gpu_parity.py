@@ -322,3 +322,71 @@ def test_screen_until_without_per_candidate_outputs_and_repeat():
     assert first[3].cpu().tolist() == [consumed, kept, batches]
     want, _ = O.topk(opf[:consumed], valid[:consumed], w.k)
     assert np.array_equal(first[2].cpu().numpy(), want)
+
+
+# --------------------------------------------------------------------------
+# Explorer proposal step (one simulated-annealing move per chain)
+# --------------------------------------------------------------------------
+
+def _gpu_sa(radices, options, program, parent, ps, kd, dd, lu, temperature, thr):
+    import torch
+
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a).astype(dt)).cuda()
+    nxt, nsc, acc = mlt.sa_step(radices, options, program, t(parent, np.int64), t(ps, np.float32),
+                                t(np.asarray(kd, np.uint32).view(np.int32), np.int32),
+                                t(np.asarray(dd, np.uint32).view(np.int32), np.int32), t(lu, np.float32),
+                                temperature, thr)
+    mlt.sync_status()
+    return nxt.cpu().numpy(), nsc.cpu().numpy(), acc.cpu().numpy()
+
+
+def test_sa_step_hand_worked_on_gpu():
+    from conftest import floats, golden, slots_to_nodes
+
+    g = golden("sa_step.json")
+    prog = np.zeros(len(g["program"]), mlt.OP_DTYPE)
+    for i, (op, a, b, c) in enumerate(g["program"]):
+        prog[i] = (op, a, b, c)
+    mlt.set_num_features(2)
+    mlt.load_ensemble(mlt.MLT_MODEL_V, slots_to_nodes(g["V"], mlt.NODE_DTYPE), 1, 1)
+    mlt.load_ensemble(mlt.MLT_MODEL_P, slots_to_nodes(g["P"], mlt.NODE_DTYPE), 1, 1)
+    for case in g["cases"]:
+        nxt, nsc, acc = _gpu_sa(g["radices"], np.array(g["options"], np.float32), prog, g["parent"],
+                                floats(g["parent_score"]), g["knob_draw"], g["digit_draw"], floats(g["log_u"]),
+                                case["temperature"], g["thr"])
+        assert nxt.tolist() == case["next"]
+        assert_same_bits(nsc, floats(case["score"]), "chain scores")
+        assert acc.tolist() == case["accepted"]
+
+
+def test_sa_chains_match_oracle_over_three_steps():
+    w = W.make_workload(4, seed=1, n=1000)
+    d = w.decoder
+    mlt.load_workload_models(w)
+    rng = np.random.default_rng(12)
+    m = 6000
+    parent = rng.integers(0, d.space, size=m).astype(np.int64)
+    parent[::97] = -1  # inactive chains
+    ps = np.full(m, -np.inf, np.float32)
+    for step, temperature in enumerate([2.0, 1.0, 0.25]):
+        kd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+        dd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+        lu = np.log(rng.random(m)).astype(np.float32)
+        g = _gpu_sa(d.radices, d.option_values, d.program, parent, ps, kd, dd, lu, temperature, w.thr)
+        o = O.sa_step(d.radices, d.option_values, d.program, w.v, w.p, parent, ps, kd, dd, lu, temperature, w.thr)
+        assert np.array_equal(g[0], o[0]), step
+        assert_same_bits(g[1], o[1], f"chain scores step {step}")
+        assert np.array_equal(g[2], o[2]), step
+        parent, ps = o[0], o[1]
+    assert 0 < int(g[2].sum()) < m
+
+
+def test_sa_step_reports_parent_past_the_space():
+    w = W.make_workload(4, seed=1, n=100)
+    d = w.decoder
+    mlt.load_workload_models(w)
+    with pytest.raises(mlt.MltError) as e:
+        _gpu_sa(d.radices, d.option_values, d.program, [3, d.space], [0.0, 0.0], [1, 1], [1, 1], [-1.0, -1.0],
+                1.0, w.thr)
+    assert e.value.code == -1
+    mlt.sync_status()

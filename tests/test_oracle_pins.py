@@ -283,3 +283,55 @@ def test_rerank_equals_sorted_margins(seed):
     assert final.tolist() == want + [-1] * (25 - len(want))
     for i, c in enumerate(cand):
         assert same_float(score[i], m[c] if c >= 0 else np.float32(-np.inf))
+
+
+# --------------------------------------------------------------------------
+# Explorer proposal step
+# --------------------------------------------------------------------------
+
+def _sa_fixture():
+    g = golden("sa_step.json")
+    prog = np.zeros(len(g["program"]), O.OP_DTYPE)
+    for i, (op, a, b, c) in enumerate(g["program"]):
+        prog[i] = (op, a, b, c)
+    v = (slots_to_nodes(g["V"], O.NODE_DTYPE), len(g["V"]), g["depth"])
+    p = (slots_to_nodes(g["P"], O.NODE_DTYPE), len(g["P"]), g["depth"])
+    return g, prog, v, p
+
+
+def test_sa_step_hand_worked():
+    g, prog, v, p = _sa_fixture()
+    for case in g["cases"]:
+        nxt, nsc, acc = O.sa_step(g["radices"], g["options"], prog, v, p, g["parent"], floats(g["parent_score"]),
+                                  g["knob_draw"], g["digit_draw"], floats(g["log_u"]), case["temperature"], g["thr"])
+        assert nxt.tolist() == case["next"]
+        assert same_float(nsc, floats(case["score"]))
+        assert acc.tolist() == case["accepted"]
+
+
+def test_sa_step_proposals_change_one_knob():
+    d = W.conv2d_decoder(seed=1)
+    w = W.make_workload(4, seed=1, n=2000)
+    rng = np.random.default_rng(3)
+    m = 300
+    parent = rng.integers(0, d.space, size=m)
+    ps = np.full(m, -np.inf, np.float32)  # every valid proposal is accepted
+    kd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+    dd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+    lu = np.log(rng.random(m)).astype(np.float32)
+    nxt, nsc, acc = O.sa_step(d.radices, d.option_values, d.program, w.v, w.p, parent, ps, kd, dd, lu, 1.0, w.thr)
+    pk = O.decode(d.radices, 0, 1)  # warm the library
+    for i in range(m):
+        a = O.decode(d.radices, int(parent[i]), 1)[0]
+        j = int(kd[i]) % 8
+        q = a.copy()
+        q[j] = int(dd[i]) % 8
+        qi = int(sum(int(q[t]) * 8 ** t for t in range(8)))
+        if acc[i]:
+            assert nxt[i] == qi
+            _, f = O.features(d.radices, d.option_values, d.program, qi, 1)
+            _, pf, valid, _ = O.screen_rows(f, w.v, w.p, w.thr)
+            assert valid[0] and same_float(nsc[i], pf[0])
+        else:
+            assert nxt[i] == parent[i] and np.isneginf(nsc[i])
+    del pk
