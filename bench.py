@@ -101,17 +101,35 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # the oracle on the host cores
 # ---------------------------------------------------------------------------
+def oracle_pass(w, rows: int):
+    """One whole oracle pass over the workload's first `rows` candidates:
+    (decode +) V screen + P score + top-k, single thread."""
+    import oracle as O
+
+    if w.decoder is None:
+        x = w.feats[:rows]
+    else:
+        d = w.decoder
+        _, x = O.features(d.radices, d.option_values, d.program, w.first_index, rows)
+    return O.screen(x, w.v, w.p, w.thr, w.k)
+
+
 def oracle_rate(w, budget_s: float, rows_per_call: int | None = None):
     """Single-threaded oracle throughput (candidates/s) on leading rows of
     the workload: whole oracle passes (screen + top-k) of `rows_per_call`
     rows until `budget_s` seconds have been spent."""
-    import oracle as O
-
-    n = w.n if rows_per_call is None else min(w.n, rows_per_call)
+    if rows_per_call is None:
+        # whole workload if one pass fits the budget, else a leading slice
+        probe = min(w.n, 1024)
+        t0 = time.perf_counter()
+        oracle_pass(w, probe)
+        per_row = (time.perf_counter() - t0) / probe
+        rows_per_call = int(max(probe, budget_s / 4 / max(per_row, 1e-9)))
+    n = min(w.n, rows_per_call)
     done, t0 = 0, time.perf_counter()
     calls = 0
     while True:
-        O.screen(w.feats[:n], w.v, w.p, w.thr, w.k)
+        oracle_pass(w, n)
         done += n
         calls += 1
         el = time.perf_counter() - t0
@@ -126,25 +144,27 @@ def run_reference(args):
         return 0
     from paper_2411_10764_gb300 import workloads as W
 
-    w = W.make_workload(args.config, seed=args.seed)
+    w = W.make_workload(args.config, seed=args.seed, n=args.n)
     import oracle as O
 
     O.build()
     # size one step so that warmup + steps stay near 60 s of oracle work
+    probe = min(w.n, 1024)
     t0 = time.perf_counter()
-    O.screen(w.feats[:1024], w.v, w.p, w.thr, w.k)
-    per_row = (time.perf_counter() - t0) / 1024
+    oracle_pass(w, probe)
+    per_row = (time.perf_counter() - t0) / probe
     rows = int(max(64, min(w.n, 60.0 / max(1, args.steps + args.warmup) / max(per_row, 1e-9))))
     for _ in range(args.warmup):
-        O.screen(w.feats[:rows], w.v, w.p, w.thr, w.k)
+        oracle_pass(w, rows)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        O.screen(w.feats[:rows], w.v, w.p, w.thr, w.k)
+        oracle_pass(w, rows)
         times.append(time.perf_counter() - t0)
     mean = sum(times) / len(times)
     value = rows / mean
-    sample = f"first {rows} of {w.n} candidates per step (whole oracle pass: V, P, sort)"
+    what = "decode, V, P, sort" if w.decoder is not None else "V, P, sort"
+    sample = f"first {rows} of {w.n} candidates per step (whole oracle pass: {what})"
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "candidates/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -201,16 +221,53 @@ def dram_traffic(config: int, phase: str):
     return ent.get("dram_bytes_per_launch") if ent else None
 
 
-def algorithmic_counts(w, survivors):
-    """Node visits and algorithmic HBM bytes of one step (see the design notes)."""
+def mean_path(ens, x):
+    """Mean number of split nodes a row of `x` passes through per tree
+    (the walk's node visits), counted by walking the heap-ordered trees
+    with numpy.  For full trees this is the depth."""
+    t = ens.nodes.reshape(ens.n_trees, -1)
+    feat, val, dl = t["feature"], t["value"], t["default_left"].astype(bool)
+    tree = np.arange(ens.n_trees)[None, :]
+    node = np.zeros((x.shape[0], ens.n_trees), np.int64)
+    rows = np.arange(x.shape[0])[:, None]
+    visits = 0
+    for _ in range(ens.depth):
+        f = feat[tree, node]
+        active = f >= 0
+        if not active.any():
+            break
+        xv = x[rows, np.maximum(f, 0)]
+        left = np.where(np.isnan(xv), dl[tree, node], xv < val[tree, node])
+        node = np.where(active, 2 * node + 1 + (~left), node)
+        visits += int(active.sum())
+    return visits / (x.shape[0] * ens.n_trees)
+
+
+def algorithmic_counts(w, survivors, survived_rows=None):
+    """Node visits and algorithmic HBM bytes of one step (see the design
+    notes).  Full trees: trees x depth visits per candidate; unbalanced
+    trees: trees x the mean path length over a 2,048-row sample (the P
+    pass's over the sample's survivors)."""
     c = w.cfg
-    v_visits = w.n * c.v_trees * c.v_depth
-    p_visits = survivors * c.p_trees * c.p_depth
+    if c.shape == "full":
+        v_path, p_path = float(c.v_depth), float(c.p_depth)
+    else:
+        xs = w.feats[:2048]
+        v_path = mean_path(w.v, xs)
+        keep = xs if survived_rows is None else xs[survived_rows[:xs.shape[0]]]
+        p_path = mean_path(w.p, keep if keep.shape[0] else xs)
+    v_visits = w.n * c.v_trees * v_path
+    p_visits = survivors * c.p_trees * p_path
     feat_bytes = 0 if w.feats is None else w.feats.nbytes
-    v_table = c.v_trees * (((1 << c.v_depth) - 1) * 8 + (1 << c.v_depth) * 4)
-    p_table = c.p_trees * (((1 << c.p_depth) - 1) * 8 + (1 << c.p_depth) * 4)
+    # 8 B per split node (threshold + feature), 4 B per leaf value
+    def table(ens):
+        f = ens.nodes["feature"]
+        return int((f >= 0).sum()) * 8 + int((f == -1).sum()) * 4
+
+    v_table, p_table = table(w.v), table(w.p)
     out_bytes = w.n * 8 + c.k * 8
-    return {"v_visits": v_visits, "p_visits": p_visits, "feat_bytes": feat_bytes,
+    return {"v_visits": v_visits, "p_visits": p_visits, "v_path": v_path, "p_path": p_path,
+            "feat_bytes": feat_bytes,
             "v_table_bytes": v_table, "p_table_bytes": p_table, "out_bytes": out_bytes,
             "survivor_feat_bytes": survivors * c.F * 4}
 
@@ -234,18 +291,24 @@ def run_ours(args):
     from paper_2411_10764_gb300 import workloads as W
 
     seed = args.seed + rank
-    w = W.make_workload(args.config, seed=seed)
+    w = W.make_workload(args.config, seed=seed, n=args.n)
     mlt.load_workload_models(w)
-    x = torch.from_numpy(w.feats).to(dev)
     n, k, thr = w.n, w.k, w.thr
     pv = torch.empty(n, dtype=torch.float32, device=dev)
     pf = torch.empty(n, dtype=torch.float32, device=dev)
     tk = torch.empty(k, dtype=torch.int64, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    d = w.decoder
+    x = None if d is not None else torch.from_numpy(w.feats).to(dev)
 
     def step():
-        mlt.screen(x, thr, k, pv, pf, tk, stream=stream)
+        if d is None:
+            mlt.screen(x, thr, k, pv, pf, tk, stream=stream)
+        else:
+            # knob indices decoded and featurised inside the walk kernels
+            mlt.screen_decoded(d.radices, d.option_values, d.program, w.first_index, n, thr, k,
+                               out_pvalid=pv, out_perf=pf, out_topk=tk, stream=stream)
 
     for _ in range(max(3, args.warmup)):
         flush.fill_(1.0)
@@ -304,7 +367,7 @@ def run_ours(args):
     # model A's rerank of the kept (alpha+1)N = k candidates down to N = k/2
     # (alpha = 1): 300 trees, depth <= 14 (Table 3), timed per call
     rerank = None
-    if not args.no_rerank:
+    if not args.no_rerank and x is not None:
         a = W.make_model_a(w, seed=seed)
         mlt.load_ensemble(mlt.MLT_MODEL_A, a.nodes, a.n_trees, a.depth)
         n_final = max(1, k // 2)
@@ -325,19 +388,34 @@ def run_ours(args):
         rerank = {"what": f"model A rerank of the top-{k} to {n_final}", "a_trees": a.n_trees,
                   "a_max_depth": a.depth, "a_nodes": nodes_a, "us_per_call": r0.elapsed_time(r1) * 1e3 / reps}
 
-    # end to end through the host-buffer entry point (pinned host memory)
-    hx = torch.from_numpy(w.feats).pin_memory()
+    # end to end through the host-buffer entry point (pinned host memory);
+    # a decoded workload's only input is its knob space (radices, option
+    # values, feature program), and its results are read back the same way
     hpv = torch.empty(n, dtype=torch.float32).pin_memory()
     hpf = torch.empty(n, dtype=torch.float32).pin_memory()
     htk = torch.empty(k, dtype=torch.int64).pin_memory()
     out = (hpv.numpy(), hpf.numpy(), htk.numpy())
-    hxn = hx.numpy()
+    if d is None:
+        hxn = torch.from_numpy(w.feats).pin_memory().numpy()
+        h2d_bytes = int(w.feats.nbytes)
+
+        def e2e_step():
+            mlt.screen_host(hxn, thr, k, out=out, stream=stream)
+    else:
+        h2d_bytes = int(d.radices.nbytes + d.option_values.nbytes + d.program.nbytes)
+
+        def e2e_step():
+            step()
+            hpv.copy_(pv, non_blocking=True)
+            hpf.copy_(pf, non_blocking=True)
+            htk.copy_(tk, non_blocking=True)
+            torch.cuda.current_stream(dev).synchronize()
     for _ in range(3):
-        mlt.screen_host(hxn, thr, k, out=out, stream=stream)
-    e2e_steps = max(10, min(args.steps, 200))
+        e2e_step()
+    e2e_steps = max(10, min(args.steps, 200 if n <= (1 << 20) else 10))
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
-        mlt.screen_host(hxn, thr, k, out=out, stream=stream)
+        e2e_step()
     e2e_s = (time.perf_counter() - t0) / e2e_steps
     if dist is not None:
         t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
@@ -350,7 +428,10 @@ def run_ours(args):
         return 0
 
     hbm_gbs, sm_max, peak_src = peaks()
-    cnt = algorithmic_counts(w, survivors)
+    survived = None
+    if w.cfg.shape != "full":
+        survived = torch.isfinite(pf[:2048]).cpu().numpy()
+    cnt = algorithmic_counts(w, survivors, survived)
     v_ms = phases["v_pass"] / max(calls, 1)
     p_ms = phases["p_pass"] / max(calls, 1)
     dominant = "v_pass" if v_ms >= p_ms else "p_pass"
@@ -386,7 +467,7 @@ def run_ours(args):
             "dominant_kernel_gbs": dom_bytes / (dom_ms / 1e3) / 1e9,
         },
         "e2e": {"value": world * n / e2e_s, "unit": "candidates/s",
-                "h2d_bytes_per_step": int(w.feats.nbytes),
+                "h2d_bytes_per_step": h2d_bytes,
                 "d2h_bytes_per_step": int(2 * n * 4 + k * 8)},
         "gpu_launches": int(launches),
         "rerank": rerank,
@@ -396,7 +477,7 @@ def run_ours(args):
     if not args.no_cpu_baseline:
         rate, info = oracle_rate(w, args.cpu_seconds)
         line["cpu_baseline"] = {"value": rate, "unit": "candidates/s", "cores": 1, "kind": "oracle",
-                                "sample": f"whole workload ({info['rows_per_call']} candidates) x "
+                                "sample": f"first {info['rows_per_call']} of {w.n} candidates x "
                                           f"{info['calls']} oracle passes, {info['seconds']} s, single thread"}
     print(json.dumps(line), flush=True)
     if dist is not None:
@@ -415,6 +496,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-rerank", action="store_true")
+    ap.add_argument("--n", type=int, default=None,
+                    help="candidates per batch (default: the workload's size; smaller for profiling captures)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
