@@ -298,6 +298,14 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  * to the library's choice.  Results do not depend on the shape.  Host-only. */
 int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf);
 
+/* Tuning of the deep-tree walk (ensembles deeper than 10 levels, whose
+ * nodes are read from L1/L2): candidates per CTA (32, 64, 128 or 256), lanes
+ * sharing one candidate's trees (1, 2, 4 or 8; candidates x lanes <= 256)
+ * and trees in flight per lane (4 or 8); 0 = let the library choose.  A
+ * shape that does not fit shared memory falls back to the library's choice.
+ * Results do not depend on the shape.  Host-only. */
+int mlt_tune_deep_walk(int model_id, int candidates, int lanes, int group);
+
 /* Cumulative number of GPU kernels this library has launched. */
 int64_t mlt_kernel_launches(void);
 

@@ -251,7 +251,8 @@ ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeO
   ScreenShape s = dm.kind == kTableFull
                       ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
                       : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
-  if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf)) return plan_for(dm, F, n_eff, ShapeOverride());
+  if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
+    return plan_for(dm, F, n_eff, ShapeOverride());
   return s;
 }
 
@@ -976,6 +977,22 @@ int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf) {
   g_shape[model_id].threads = threads;
   g_shape[model_id].chunk_trees = chunk_trees;
   g_shape[model_id].nbuf = nbuf;
+  return MLT_OK;
+}
+
+int mlt_tune_deep_walk(int model_id, int candidates, int lanes, int group) {
+  if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
+  if (!(candidates == 0 || candidates == 32 || candidates == 64 || candidates == 128 || candidates == 256))
+    return fail(MLT_EINVAL, "candidates must be 0, 32, 64, 128 or 256");
+  if (!(lanes == 0 || lanes == 1 || lanes == 2 || lanes == 4 || lanes == 8))
+    return fail(MLT_EINVAL, "lanes must be 0, 1, 2, 4 or 8");
+  if (!(group == 0 || group == 4 || group == 8)) return fail(MLT_EINVAL, "group must be 0, 4 or 8");
+  if (candidates && lanes && candidates * lanes > 256)
+    return fail(MLT_EINVAL, "candidates x lanes must be at most 256");
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_shape[model_id].threads = candidates;
+  g_shape[model_id].lanes = lanes;
+  g_shape[model_id].group = group;
   return MLT_OK;
 }
 

@@ -189,13 +189,17 @@ struct ScreenShape {
   int chunk_trees;
   int nbuf;
   int group;           // trees walked together per thread (ILP)
+  int lanes = 1;       // lanes sharing one candidate (compact walk; CTA = threads * lanes)
 };
 
-// Launch-shape override (mlt_tune_shape): 0 fields mean "choose".
+// Launch-shape override (mlt_tune_shape, mlt_tune_deep_walk): 0 fields mean
+// "choose".
 struct ShapeOverride {
   int threads = 0;
   int chunk_trees = 0;
   int nbuf = 0;
+  int lanes = 0;
+  int group = 0;
 };
 
 // traverse.cu

@@ -99,32 +99,81 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
   return best;  // threads == 0: nothing fits
 }
 
+// Deep-tree walk: candidates per CTA (TC), lanes per candidate (Q) and trees
+// in flight per lane (G).  Every visit waits on an L1/L2 load, so a
+// candidate's walk takes time in proportion to its trees / (Q * G), and an SM
+// finishes (resident CTAs * TC * Q * G) walks in flight at a time.  Measured
+// on GB300 (F = 256, 1,000-2,000 trees of depth <= 12): throughput grows
+// with the walks in flight up to about 3,072 per SM and falls beyond it, as
+// the trees in flight crowd L1.  So the rule minimises
+//   (candidates per SM) / (walks in flight, counted up to 3,072 and
+//                          discounted by a quarter of any excess)
+// where resident CTAs are limited by shared memory (F * TC * 4 bytes of
+// features), 2,048 threads, registers (48 a thread at G = 4, 64 at G = 8)
+// and the tiles the batch gives each SM.  Ties go to fewer lanes (fewer
+// bank conflicts on the feature gathers), then to larger CTAs.
 ScreenShape plan_compact(int F, long long n_eff, int sms, int optin, const ShapeOverride& ov) {
+  constexpr double kSaturation = 3072.0;
   ScreenShape best{};
   double best_cost = 1e300;
   if (sms < 1) sms = 1;
   if (n_eff < 1) n_eff = 1;
-  for (int tc : {256, 128, 64, 32}) {
-    if (ov.threads && tc != ov.threads) continue;
-    const size_t smem = compact_smem_bytes(F, tc);
-    if (smem + kStaticSmem > static_cast<size_t>(optin)) continue;
-    const int ctas_sm = static_cast<int>(std::min<size_t>(
-        {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / tc), 32}));
-    if (ctas_sm < 1) continue;
-    const long long tiles = (n_eff + tc - 1) / tc;
-    const long long tiles_sm = (tiles + sms - 1) / sms;
-    const int resident = static_cast<int>(std::min<long long>(ctas_sm, tiles_sm));
-    const double eff = std::min(1.0, resident * tc / 32 * 4 / 64.0);
-    const double cost = static_cast<double>(tiles_sm) * tc / eff;
-    if (cost < best_cost) {
-      best_cost = cost;
-      best.threads = tc;
-      best.smem = smem;
+  for (int q : {1, 2, 4, 8}) {
+    if (ov.lanes && q != ov.lanes) continue;
+    for (int tc : {256, 128, 64, 32}) {
+      if (ov.threads && tc != ov.threads) continue;
+      const int threads = tc * q;
+      if (threads > 256) continue;
+      const size_t smem = compact_smem_bytes(F, tc);
+      if (smem + kStaticSmem > static_cast<size_t>(optin)) continue;
+      for (int g : {8, 4}) {
+        if (ov.group && g != ov.group) continue;
+        const int regs = g == 8 ? 64 : 48;
+        const int ctas_sm = static_cast<int>(std::min<size_t>(
+            {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / threads),
+             static_cast<size_t>(65536 / (threads * regs)), 32}));
+        if (ctas_sm < 1) continue;
+        const long long tiles = (n_eff + tc - 1) / tc;
+        const long long tiles_sm = (tiles + sms - 1) / sms;
+        const int resident = static_cast<int>(std::min<long long>(ctas_sm, tiles_sm));
+        const double inflight = static_cast<double>(resident) * threads * g;
+        const double eff = inflight <= kSaturation ? inflight
+                                                   : std::max(kSaturation - 0.25 * (inflight - kSaturation), 256.0);
+        const double cost = static_cast<double>(tiles_sm) * tc / eff;
+        if (cost < best_cost * (1.0 - 1e-9)) {
+          best_cost = cost;
+          best.threads = tc;
+          best.lanes = q;
+          best.group = g;
+          best.smem = smem;
+        }
+      }
     }
   }
-  best.group = 8;
   return best;
 }
+
+namespace {
+using CompactKernel = void (*)(TraverseArgs);
+CompactKernel compact_kernel(int group, int lanes) {
+  if (group == 8) {
+    switch (lanes) {
+      case 1: return k_traverse_compact<8, 1>;
+      case 2: return k_traverse_compact<8, 2>;
+      case 4: return k_traverse_compact<8, 4>;
+      case 8: return k_traverse_compact<8, 8>;
+    }
+  } else if (group == 4) {
+    switch (lanes) {
+      case 1: return k_traverse_compact<4, 1>;
+      case 2: return k_traverse_compact<4, 2>;
+      case 4: return k_traverse_compact<4, 4>;
+      case 8: return k_traverse_compact<4, 8>;
+    }
+  }
+  return nullptr;
+}
+}  // namespace
 
 cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, const ScreenShape& shape,
                             long long n_tiles, cudaStream_t st) {
@@ -141,10 +190,12 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     e = launch_pdl(k, grid, block, shape.smem, st, args);
     if (e != cudaSuccess) return e;
   } else {
-    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    CompactKernel k = compact_kernel(shape.group, shape.lanes);
+    if (k == nullptr) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_traverse_compact<8>, grid, block, shape.smem, st, args);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, args);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

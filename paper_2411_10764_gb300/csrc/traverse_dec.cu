@@ -30,6 +30,27 @@ FullDecKernel full_dec_kernel(int d) {
   }
 }
 
+using CompactDecKernel = void (*)(TraverseArgs, DecodeParams);
+
+CompactDecKernel compact_dec_kernel(int group, int lanes) {
+  if (group == 8) {
+    switch (lanes) {
+      case 1: return k_traverse_compact_dec<8, 1>;
+      case 2: return k_traverse_compact_dec<8, 2>;
+      case 4: return k_traverse_compact_dec<8, 4>;
+      case 8: return k_traverse_compact_dec<8, 8>;
+    }
+  } else if (group == 4) {
+    switch (lanes) {
+      case 1: return k_traverse_compact_dec<4, 1>;
+      case 2: return k_traverse_compact_dec<4, 2>;
+      case 4: return k_traverse_compact_dec<4, 4>;
+      case 8: return k_traverse_compact_dec<4, 8>;
+    }
+  }
+  return nullptr;
+}
+
 // One thread per candidate: decode into a shared-memory column, then write
 // the rows out coalesced.
 __global__ void __launch_bounds__(256)
@@ -78,11 +99,12 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     e = launch_pdl(k, grid, block, shape.smem, st, args, dec);
     if (e != cudaSuccess) return e;
   } else {
-    cudaError_t e = cudaFuncSetAttribute(k_traverse_compact_dec<8>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+    CompactDecKernel k = compact_dec_kernel(shape.group, shape.lanes);
+    if (k == nullptr) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_traverse_compact_dec<8>, grid, block, shape.smem, st, args, dec);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, args, dec);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

@@ -272,8 +272,11 @@ __device__ __forceinline__ void scan_tiles(const uint32_t* counts, uint32_t* off
     for (int i = tid; i < kTopBins; i += T) st->hist[i] = 0u;
   (void)nw;
 }
+// Threads [0, tc) hold the tile's candidates (tc = candidates per CTA, a
+// multiple of 32); every thread of the CTA calls this.
 __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_t* rowidx,
-                                            long long tile0, int rows_here, long long count, float acc) {
+                                            long long tile0, int rows_here, long long count, float acc,
+                                            int tc) {
   const int tid = threadIdx.x;
   const bool in = tid < rows_here;
   if (a.p_pass) {
@@ -303,7 +306,7 @@ __device__ __forceinline__ void finish_tile(const TraverseArgs& a, const uint32_
   const unsigned ball = __ballot_sync(0xFFFFFFFFu, valid);
   const int warp = tid >> 5;
   if ((tid & 31) == 0) {
-    if (tile0 + warp * 32 < count) a.masks[(tile0 >> 5) + warp] = ball;
+    if (warp * 32 < tc && tile0 + warp * 32 < count) a.masks[(tile0 >> 5) + warp] = ball;
     warp_count[warp] = __popc(ball);
   }
   __shared__ unsigned is_last;
@@ -519,7 +522,7 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     if (tid == 0 && c + a.nbuf < n_chunks) issue(c + a.nbuf, b);
   }
   pdl_trigger();
-  finish_tile(a, rowidx, tile0, rows_here, count, acc);
+  finish_tile(a, rowidx, tile0, rows_here, count, acc, TC);
 }
 
 template <int D, int G>
@@ -536,14 +539,25 @@ __global__ void __launch_bounds__(256)
 // ---------------------------------------------------------------------------
 // Compact-table walk (nodes from global memory)
 // ---------------------------------------------------------------------------
+// Deep trees do not fit shared memory, so their nodes come from L1/L2 and
+// every visit is a dependent load: the walk is latency-bound and needs many
+// walks in flight per SM.  A wide feature row (1 KB at F = 256) leaves room
+// for few candidates per SM, so Q lanes share one candidate: lane q of a
+// candidate walks trees t0 + g*Q + q (g < G), and the G*Q leaves of each
+// group are added in tree order through warp shuffles -- the same sequential
+// fp32 sum as a single walker.  A warp holds 32/Q candidates.
+//
+// Shared memory: features [F][TC] (TC = candidates per CTA = blockDim / Q),
+// then the survivor positions [TC] and the candidates' sums [TC].
 __host__ __device__ inline size_t compact_smem_bytes(int F, int TC) {
-  return align_up(static_cast<size_t>(F) * TC * 4, 128) + align_up(static_cast<size_t>(TC) * 4, 128);
+  return align_up(static_cast<size_t>(F) * TC * 4, 128) + 2 * align_up(static_cast<size_t>(TC) * 4, 128);
 }
 
-template <int G>
+template <int G, int Q>
 __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, const DecodeParams* dec) {
   extern __shared__ __align__(128) unsigned char smem[];
-  const int TC = blockDim.x;
+  constexpr int kCpw = 32 / Q;  // candidates per warp
+  const int TC = blockDim.x / Q;
   const int tid = threadIdx.x;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
   pdl_wait();
@@ -553,69 +567,83 @@ __device__ __forceinline__ void traverse_compact_body(const TraverseArgs& a, con
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
 
   float* xs = reinterpret_cast<float*>(smem);
-  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + align_up(static_cast<size_t>(a.F) * TC * 4, 128));
+  const size_t rows_off = align_up(static_cast<size_t>(a.F) * TC * 4, 128);
+  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + rows_off);
+  float* sums = reinterpret_cast<float*>(smem + rows_off + align_up(static_cast<size_t>(TC) * 4, 128));
   if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
-  // feature rows are read once; the node tables are re-read by every tile
-  __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC, true));
+  // threads [0, TC) stage one row each; feature rows are read once, the node
+  // tables are re-read by every tile
+  __syncthreads_or(tid < TC && stage_row(a, dec, xs, rowidx, tile0, rows_here, TC, true));
 
-  const uint32_t* offs = reinterpret_cast<const uint32_t*>(a.table);
-  const uint2* recs =
-      reinterpret_cast<const uint2*>(a.table + align_up(static_cast<size_t>(a.n_trees) * 4, 16));
-  const unsigned long long keep = policy_evict_last();
+  const int lane = tid & 31, warp = tid >> 5;
+  const int cl = lane % kCpw;       // candidate within the warp
+  const int q = lane / kCpw;        // this lane's share of each tree group
+  const int c = warp * kCpw + cl;   // candidate within the tile
   float acc = 0.0f;
-  const int steps = a.max_depth + 1;
-  for (int t = 0; t < a.n_trees; t += G) {
-    const uint2* tr[G];
-    uint32_t j[G];
-    float leaf[G];
-    bool live[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      live[g] = (t + g) < a.n_trees;
-      tr[g] = recs + (live[g] ? __ldg(offs + t + g) : 0u);
-      j[g] = 0;
-      leaf[g] = 0.0f;
-    }
-    for (int s = 0; s < steps; ++s) {
-      // all G node loads first (a finished walk re-reads its leaf: the
-      // address stays inside its tree), then the decisions
+  if (warp * kCpw < rows_here) {    // warp-uniform: a warp past the rows idles
+    const uint32_t* offs = reinterpret_cast<const uint32_t*>(a.table);
+    const uint2* recs =
+        reinterpret_cast<const uint2*>(a.table + align_up(static_cast<size_t>(a.n_trees) * 4, 16));
+    const unsigned long long keep = policy_evict_last();
+    const float* xc = xs + c;
+    const int steps = a.max_depth + 1;
+    for (int t0 = 0; t0 < a.n_trees; t0 += G * Q) {
+      const uint2* tr[G];
+      uint32_t j[G];
+      bool live[G];
       uint2 r[G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) r[g] = ldg_u2_hint(tr[g] + j[g], keep);
-      bool any = false;
+      for (int g = 0; g < G; ++g) {
+        const int t = t0 + g * Q + q;
+        live[g] = t < a.n_trees;
+        tr[g] = recs + (live[g] ? __ldg(offs + t) : 0u);
+        j[g] = 0;
+      }
+      for (int s = 0; s < steps; ++s) {
+        // all G node loads, then the decisions; a walk at its leaf stays
+        // there (its record is re-read, a leaf's feature field is 0)
+#pragma unroll
+        for (int g = 0; g < G; ++g) r[g] = ldg_u2_hint(tr[g] + j[g], keep);
+        bool any = false;
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          const uint32_t meta = r[g].y;
+          const float x = xc[(meta & kCompactFeatureMask) * TC];
+          uint32_t right = x >= __uint_as_float(r[g].x) ? 1u : 0u;
+          if ((x != x) && !(meta & kMetaDefaultLeft)) right = 1u;
+          const bool move = live[g] && !(meta & kMetaLeaf);
+          j[g] = move ? ((meta >> kCompactChildShift) & kCompactChildMask) + right : j[g];
+          any |= move;
+        }
+        if (!__any_sync(0xFFFFFFFFu, any)) break;  // every walk of the warp is at a leaf
+      }
+      // r[g] is each walk's leaf record.  Tree t0 + g*Q + qq of candidate c
+      // sits in lane qq*kCpw + cl: add them in tree order.
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        if (!live[g]) continue;
-        if (r[g].y & kMetaLeaf) {
-          leaf[g] = __uint_as_float(r[g].x);
-          live[g] = false;
-        } else {
-          const float x = xs[(r[g].y & kCompactFeatureMask) * TC + tid];
-          uint32_t right = x >= __uint_as_float(r[g].x) ? 1u : 0u;
-          if ((x != x) && !(r[g].y & kMetaDefaultLeft)) right = 1u;
-          j[g] = ((r[g].y >> kCompactChildShift) & kCompactChildMask) + right;
-          any = true;
+#pragma unroll
+        for (int qq = 0; qq < Q; ++qq) {
+          const float v = __shfl_sync(0xFFFFFFFFu, __uint_as_float(r[g].x), qq * kCpw + cl);
+          if (t0 + g * Q + qq < a.n_trees) acc += v;
         }
       }
-      if (!__any_sync(0xFFFFFFFFu, any)) break;  // every walk of the warp is at a leaf
     }
-#pragma unroll
-    for (int g = 0; g < G; ++g)
-      if (t + g < a.n_trees) acc += leaf[g];
   }
+  if (q == 0) sums[c] = acc;
+  __syncthreads();
   pdl_trigger();
-  finish_tile(a, rowidx, tile0, rows_here, count, acc);
+  finish_tile(a, rowidx, tile0, rows_here, count, tid < TC ? sums[tid] : 0.0f, TC);
 }
 
-template <int G>
+template <int G, int Q>
 __global__ void __launch_bounds__(256) k_traverse_compact(const __grid_constant__ TraverseArgs a) {
-  traverse_compact_body<G>(a, nullptr);
+  traverse_compact_body<G, Q>(a, nullptr);
 }
 
-template <int G>
+template <int G, int Q>
 __global__ void __launch_bounds__(256)
     k_traverse_compact_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
-  traverse_compact_body<G>(a, &d);
+  traverse_compact_body<G, Q>(a, &d);
 }
 
 }  // namespace walk

@@ -129,3 +129,18 @@ def test_decoder_validation(L):
     r2[0] = 0
     assert call(r2, prog, 0, 1) == -1
     assert call(r, prog, 0, 1, F=257) == -1
+
+
+@pytest.mark.parametrize("args", [(0, 48, 1, 4), (0, 64, 3, 4), (0, 64, 8, 4), (0, 64, 4, 2), (5, 64, 4, 4)])
+def test_deep_walk_tuning_rejects(args):
+    from paper_2411_10764_gb300 import mlt
+
+    with pytest.raises(mlt.MltError):
+        mlt.tune_deep_walk(*args)
+
+
+def test_deep_walk_tuning_accepts_and_releases():
+    from paper_2411_10764_gb300 import mlt
+
+    mlt.tune_deep_walk(mlt.MLT_MODEL_P, 64, 4, 8)
+    mlt.tune_deep_walk(mlt.MLT_MODEL_P)

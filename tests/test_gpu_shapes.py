@@ -1,0 +1,89 @@
+"""GPU parity for every launch shape of the walk kernels: results may not
+depend on the shape (candidates per CTA, tree chunking, lanes per candidate,
+trees in flight).  Each shape is forced through the tuning calls and
+compared bit for bit with the oracle on a batch that ends on a ragged tile."""
+import dataclasses
+
+import pytest
+
+from paper_2411_10764_gb300 import mlt
+from paper_2411_10764_gb300 import workloads as W
+from screening import assert_parity, gpu_screen, oracle_screen
+
+pytestmark = pytest.mark.gpu
+
+_ORACLE = {}
+
+
+def _expected(key, w):
+    if key not in _ORACLE:
+        _ORACLE[key] = oracle_screen(w)
+    return _ORACLE[key]
+
+
+@pytest.fixture(scope="module")
+def deep():
+    """Workload 5's shape at 3,001 candidates: 1,000 / 2,000 unbalanced trees
+    of depth <= 12 on 256 features, 30 % missing values (compact tables)."""
+    return W.make_workload(5, seed=3, n=3001)
+
+
+@pytest.fixture(scope="module")
+def deep_decoded():
+    """The conv2d knob space with unbalanced depth-12 V and P ensembles:
+    the deep walk building features from candidate indices."""
+    w = W.make_workload(4, seed=2, n=3001)
+    th = W._RangeThresholds(w.decoder.ranges)
+    v = W.make_ensemble(w.cfg, "V", th, 5, n_trees=120, depth=12, split_prob=0.85, shape="unbalanced")
+    p = W.make_ensemble(w.cfg, "P", th, 6, n_trees=200, depth=12, split_prob=0.85, shape="unbalanced")
+    return dataclasses.replace(w, v=v, p=p)
+
+
+@pytest.fixture(scope="module")
+def full():
+    return W.make_workload(2, seed=5, n=5001)
+
+
+def _release():
+    for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
+        mlt.tune_shape(m)
+        mlt.tune_deep_walk(m)
+
+
+DEEP_SHAPES = [(c, q, g) for c in (32, 64, 128, 256) for q in (1, 2, 4, 8) for g in (4, 8) if c * q <= 256]
+
+
+@pytest.mark.parametrize("cand,lanes,group", DEEP_SHAPES)
+def test_deep_walk_every_shape(deep, cand, lanes, group):
+    try:
+        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
+            mlt.tune_deep_walk(m, cand, lanes, group)
+        got = gpu_screen(deep)
+    finally:
+        _release()
+    assert_parity(got, _expected("deep", deep))
+
+
+@pytest.mark.parametrize("cand,lanes,group", [(32, 8, 4), (64, 4, 8), (128, 1, 8), (32, 2, 8)])
+def test_deep_walk_decoded_shapes(deep_decoded, cand, lanes, group):
+    try:
+        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
+            mlt.tune_deep_walk(m, cand, lanes, group)
+        got = gpu_screen(deep_decoded)
+    finally:
+        _release()
+    assert_parity(got, _expected("deep_decoded", deep_decoded))
+
+
+FULL_SHAPES = [(t, c, b) for t in (32, 64, 128, 256) for c in (1, 2, 4, 8, 16) for b in (2, 3)]
+
+
+@pytest.mark.parametrize("threads,chunk,nbuf", FULL_SHAPES)
+def test_full_walk_every_shape(full, threads, chunk, nbuf):
+    try:
+        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
+            mlt.tune_shape(m, threads, chunk, nbuf)
+        got = gpu_screen(full)
+    finally:
+        _release()
+    assert_parity(got, _expected("full", full))
