@@ -247,12 +247,17 @@ int check_models(int dev) {
   return MLT_OK;
 }
 
-ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov) {
+// v_pass: n_eff is the exact number of candidates (full tables then get
+// tiles balanced over the SMs); otherwise it is an estimate of the
+// survivors.
+ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov, bool v_pass) {
   ScreenShape s = dm.kind == kTableFull
                       ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
                       : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
   if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
-    return plan_for(dm, F, n_eff, ShapeOverride());
+    return plan_for(dm, F, n_eff, ShapeOverride(), v_pass);
+  if (v_pass && dm.kind == kTableFull && ov.threads == 0)
+    s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count());
   return s;
 }
 
@@ -429,8 +434,8 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
   // the P pass walks the survivors; plan it for about half the batch
-  const ScreenShape sv = plan_for(V, g_F, n, g_shape[MLT_MODEL_V]);
-  const ScreenShape sp = plan_for(P, g_F, (n + 1) / 2, g_shape[MLT_MODEL_P]);
+  const ScreenShape sv = plan_for(V, g_F, n, g_shape[MLT_MODEL_V], true);
+  const ScreenShape sp = plan_for(P, g_F, (n + 1) / 2, g_shape[MLT_MODEL_P], false);
   if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
   TraverseArgs a{};
   a.feats = feats;
@@ -543,8 +548,8 @@ int run_stream(cudaStream_t st, const float* feats, const DecodeParams* dec0, lo
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
   const long long per = std::min(batch, std::max(1LL, n_total));
-  const ScreenShape sv = plan_for(V, g_F, per, g_shape[MLT_MODEL_V]);
-  const ScreenShape sp = plan_for(P, g_F, (per + 1) / 2, g_shape[MLT_MODEL_P]);
+  const ScreenShape sv = plan_for(V, g_F, per, g_shape[MLT_MODEL_V], true);
+  const ScreenShape sp = plan_for(P, g_F, (per + 1) / 2, g_shape[MLT_MODEL_P], false);
   if (sv.threads == 0 || sp.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
   MLT_CUDA(cudaMemsetAsync(s.state, 0, sizeof(SelectState), st), "reset selection state");
   MLT_CUDA(cudaMemsetAsync(ss, 0, sizeof(StreamState), st), "reset stream state");

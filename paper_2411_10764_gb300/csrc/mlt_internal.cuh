@@ -181,6 +181,7 @@ struct TraverseArgs {
   // batched accumulation (null: a single batch)
   StreamState* stream;
   long long pos_base;      // position of the batch's first candidate in the call
+  int p_wave;              // full-table P pass: CTAs one wave holds (0: the grid)
 };
 
 struct ScreenShape {
@@ -190,6 +191,7 @@ struct ScreenShape {
   int nbuf;
   int group;           // trees walked together per thread (ILP)
   int lanes = 1;       // lanes sharing one candidate (compact walk; CTA = threads * lanes)
+  int p_grid = 0;      // full-table P pass: CTAs one wave holds (resident per SM x SMs)
 };
 
 // Launch-shape override (mlt_tune_shape, mlt_tune_deep_walk): 0 fields mean
@@ -208,6 +210,10 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, 
                       int device_smem_optin, const ShapeOverride& ov);
 ScreenShape plan_compact(int F, long long n_eff, int sms, int device_smem_optin,
                          const ShapeOverride& ov);
+// V pass over n known candidates: the smallest multiple of 32 candidates
+// per CTA (at least 64) that leaves the busiest SM no more tiles than `s`
+// does, so the tiles spread evenly over the SMs.
+ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms);
 cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args,
                             const ScreenShape& shape, long long n_tiles, cudaStream_t st);
 // traverse_dec.cu

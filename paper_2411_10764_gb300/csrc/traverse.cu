@@ -93,10 +93,24 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
         best.nbuf = nb;
         best.group = group;
         best.smem = smem;
+        best.p_grid = sms * resident(smem, tc);
       }
     }
   }
   return best;  // threads == 0: nothing fits
+}
+
+ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms) {
+  if (s.threads == 0 || n <= 0 || sms < 1) return s;
+  const long long tiles_sm = ((n + s.threads - 1) / s.threads + sms - 1) / sms;
+  const long long per_tile = (n + sms * tiles_sm - 1) / (sms * tiles_sm);
+  const int tc = static_cast<int>(std::min<long long>(s.threads, std::max<long long>(32, (per_tile + 31) / 32 * 32)));
+  // below two warps per CTA the table stream, not the walk, sets the pace
+  if (tc < 64 || tc == s.threads) return s;
+  ScreenShape b = s;
+  b.threads = tc;
+  b.smem = full_smem_bytes(F, tc, s.nbuf, static_cast<uint32_t>(s.chunk_trees) * tree_bytes);
+  return b;
 }
 
 // Deep-tree walk: candidates per CTA (TC), lanes per candidate (Q) and trees
@@ -178,7 +192,15 @@ CompactKernel compact_kernel(int group, int lanes) {
 cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, const ScreenShape& shape,
                             long long n_tiles, cudaStream_t st) {
   if (n_tiles <= 0) return cudaSuccess;
-  const dim3 grid(static_cast<unsigned>(n_tiles)), block(shape.threads);
+  // full-table P pass: whole waves of CTAs, the survivors split evenly over
+  // them on the device (CTAs without rows exit at once)
+  TraverseArgs a = args;
+  long long ctas = n_tiles;
+  if (args.p_pass && m.kind == kTableFull && shape.p_grid > 0) {
+    a.p_wave = shape.p_grid;
+    ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
+  }
+  const dim3 grid(static_cast<unsigned>(ctas)), block(shape.threads);
   if (m.kind == kTableFull) {
     FullKernel k = shape.group == 8   ? full_kernel<8>(m.depth)
                    : shape.group == 4 ? full_kernel<4>(m.depth)
@@ -187,7 +209,7 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, block, shape.smem, st, args);
+    e = launch_pdl(k, grid, block, shape.smem, st, a);
     if (e != cudaSuccess) return e;
   } else {
     CompactKernel k = compact_kernel(shape.group, shape.lanes);
@@ -195,7 +217,7 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, args);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, a);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

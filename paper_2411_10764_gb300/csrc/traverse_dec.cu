@@ -4,6 +4,8 @@
 // ML^2Tuner Sec. 2: the explorer enumerates the search space of
 // configurations; Appendix A.2: the knobs are tiling sizes and virtual-thread
 // counts; Table 5: derived (hidden) features.
+#include <algorithm>
+
 #include "walk.cuh"
 
 namespace mlt {
@@ -87,7 +89,15 @@ __global__ void __launch_bounds__(256)
 cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, const DecodeParams& dec,
                                 const ScreenShape& shape, long long n_tiles, cudaStream_t st) {
   if (n_tiles <= 0) return cudaSuccess;
-  const dim3 grid(static_cast<unsigned>(n_tiles)), block(shape.threads);
+  // full-table P pass: whole waves of CTAs, the survivors split evenly over
+  // them on the device (CTAs without rows exit at once)
+  TraverseArgs a = args;
+  long long ctas = n_tiles;
+  if (args.p_pass && m.kind == kTableFull && shape.p_grid > 0) {
+    a.p_wave = shape.p_grid;
+    ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
+  }
+  const dim3 grid(static_cast<unsigned>(ctas)), block(shape.threads);
   if (m.kind == kTableFull) {
     FullDecKernel k = shape.group == 8   ? full_dec_kernel<8>(m.depth)
                       : shape.group == 4 ? full_dec_kernel<4>(m.depth)
@@ -96,7 +106,7 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, block, shape.smem, st, args, dec);
+    e = launch_pdl(k, grid, block, shape.smem, st, a, dec);
     if (e != cudaSuccess) return e;
   } else {
     CompactDecKernel k = compact_dec_kernel(shape.group, shape.lanes);
@@ -104,7 +114,7 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, args, dec);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, a, dec);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();

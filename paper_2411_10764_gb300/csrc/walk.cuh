@@ -451,6 +451,41 @@ __host__ __device__ inline size_t full_smem_bytes(int F, int TC, int nbuf, uint3
   return align_up(full_smem_tbuf_off(F, TC) + static_cast<size_t>(nbuf) * chunk_bytes, 16) + 8 * 4;
 }
 
+// Even split of `len` items into `parts` contiguous pieces whose sizes
+// differ by at most one; piece i starts at split_start(len, parts, i).  The
+// survivor count is a 32-bit value, so 32-bit arithmetic suffices (a 64-bit
+// division would become a call inside the kernel).
+__device__ __forceinline__ uint32_t split_start(uint32_t len, uint32_t parts, uint32_t i) {
+  const uint32_t base = len / parts, rem = len % parts;
+  return i * base + min(i, rem);
+}
+
+// The tile of a CTA.  V pass: candidates [blockIdx.x * TC, +TC).  P pass:
+// the S survivors are split evenly into A tiles of at most TC rows, A a
+// multiple of `per_wave` (the CTAs one wave holds, a.p_wave) unless S is
+// small, then one tile per 32 rows at most -- so every SM gets the same
+// share whatever S turns out to be.  CTAs past A have no tile (len 0).
+__device__ __forceinline__ void cta_tile(const TraverseArgs& a, long long count, int TC, long long* tile0,
+                                         int* len) {
+  if (!a.p_pass) {
+    *tile0 = static_cast<long long>(blockIdx.x) * TC;
+    *len = static_cast<int>(max(0LL, min(static_cast<long long>(TC), count - *tile0)));
+    return;
+  }
+  const uint32_t S = static_cast<uint32_t>(count);
+  const uint32_t wave = a.p_wave > 0 ? static_cast<uint32_t>(a.p_wave) : gridDim.x;
+  const uint32_t waves = (S + static_cast<uint32_t>(TC) * wave - 1) / (static_cast<uint32_t>(TC) * wave);
+  const uint32_t tiles = min(min(waves * wave, (S + 31u) / 32u), gridDim.x);
+  if (blockIdx.x >= tiles) {
+    *tile0 = count;
+    *len = 0;
+    return;
+  }
+  const uint32_t lo = split_start(S, tiles, blockIdx.x);
+  *tile0 = lo;
+  *len = static_cast<int>(split_start(S, tiles, blockIdx.x + 1) - lo);
+}
+
 template <int D, int G>
 __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
   extern __shared__ __align__(128) unsigned char smem[];
