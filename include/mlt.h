@@ -291,20 +291,22 @@ int mlt_profile_phases(int enable);
  * *n_calls_out receives the number of recorded calls.  Clears the records. */
 int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
 
-/* Tuning: fix the launch shape of the walk over model `model_id`'s trees:
- * candidates per CTA (threads: 32, 64, 128 or 256), trees per shared-memory
- * chunk (1, 2, 4, 8 or 16) and chunk buffers (2 or 3); 0 = let the library
- * choose (the default).  A shape that does not fit shared memory falls back
- * to the library's choice.  Results do not depend on the shape.  Host-only. */
-int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf);
-
-/* Tuning of the deep-tree walk (ensembles deeper than 10 levels, whose
- * nodes are read from L1/L2): candidates per CTA (32, 64, 128 or 256), lanes
- * sharing one candidate's trees (1, 2, 4 or 8; candidates x lanes <= 256)
- * and trees in flight per lane (4 or 8); 0 = let the library choose.  A
- * shape that does not fit shared memory falls back to the library's choice.
- * Results do not depend on the shape.  Host-only. */
-int mlt_tune_deep_walk(int model_id, int candidates, int lanes, int group);
+/* Tuning: fix the launch shape of the tree walk over model `model_id`'s
+ * trees (0 in any field = let the library choose it):
+ *   candidates   candidates per CTA: a multiple of 32, 32 .. 256
+ *   splits       threads sharing one candidate's trees: 1, 2 or 4 for
+ *                ensembles of depth <= 10 (groups of warps, leaves summed
+ *                in tree order through shared memory), 1, 2, 4 or 8 for
+ *                deeper ones (lanes of a warp, summed through shuffles);
+ *                candidates x splits <= 256
+ *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10),
+ *                4 or 8 (deeper)
+ *   chunk_trees  trees per shared-memory chunk, 1, 2, 4, 8 or 16 (depth
+ *                <= 10 only)
+ *   nbuf         chunk buffers, 2 or 3 (depth <= 10 only)
+ * A shape that does not fit shared memory falls back to the library's
+ * choice.  Results never depend on the shape.  Host-only. */
+int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf);
 
 /* Cumulative number of GPU kernels this library has launched. */
 int64_t mlt_kernel_launches(void);

@@ -247,17 +247,17 @@ int check_models(int dev) {
   return MLT_OK;
 }
 
-// v_pass: n_eff is the exact number of candidates (full tables then get
-// tiles balanced over the SMs); otherwise it is an estimate of the
-// survivors.
+// v_pass: n_eff is the exact number of candidates; otherwise it is an
+// estimate of the survivors.  Full-table tiles are balanced over the SMs.
 ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov, bool v_pass) {
   ScreenShape s = dm.kind == kTableFull
                       ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
                       : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
   if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
     return plan_for(dm, F, n_eff, ShapeOverride(), v_pass);
-  if (v_pass && dm.kind == kTableFull && ov.threads == 0)
-    s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count());
+  // the P pass splits its survivors evenly over the CTAs on the device, so
+  // its CTA size is balanced for the estimate as well
+  if (dm.kind == kTableFull && ov.threads == 0) s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count());
   return s;
 }
 
@@ -970,34 +970,26 @@ int mlt_phase_times(float* out_ms, int n_phases, int64_t* n_calls_out) {
   return MLT_OK;
 }
 
-int mlt_tune_shape(int model_id, int threads, int chunk_trees, int nbuf) {
+int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf) {
   if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
-  if (!(threads == 0 || threads == 32 || threads == 64 || threads == 128 || threads == 256))
-    return fail(MLT_EINVAL, "threads must be 0, 32, 64, 128 or 256");
+  if (candidates < 0 || candidates > 256 || candidates % 32 != 0)
+    return fail(MLT_EINVAL, "candidates must be 0 or a multiple of 32 up to 256");
+  if (!(splits == 0 || splits == 1 || splits == 2 || splits == 4 || splits == 8))
+    return fail(MLT_EINVAL, "splits must be 0, 1, 2, 4 or 8");
+  if (!(group == 0 || group == 2 || group == 4 || group == 8)) return fail(MLT_EINVAL, "group must be 0, 2, 4 or 8");
   if (!(chunk_trees == 0 || chunk_trees == 1 || chunk_trees == 2 || chunk_trees == 4 || chunk_trees == 8 ||
         chunk_trees == 16))
     return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8 or 16");
   if (!(nbuf == 0 || nbuf == 2 || nbuf == 3)) return fail(MLT_EINVAL, "nbuf must be 0, 2 or 3");
+  if (candidates && splits && candidates * splits > 256)
+    return fail(MLT_EINVAL, "candidates x splits must be at most 256");
   std::lock_guard<std::mutex> lk(g_mu);
-  g_shape[model_id].threads = threads;
-  g_shape[model_id].chunk_trees = chunk_trees;
-  g_shape[model_id].nbuf = nbuf;
-  return MLT_OK;
-}
-
-int mlt_tune_deep_walk(int model_id, int candidates, int lanes, int group) {
-  if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
-  if (!(candidates == 0 || candidates == 32 || candidates == 64 || candidates == 128 || candidates == 256))
-    return fail(MLT_EINVAL, "candidates must be 0, 32, 64, 128 or 256");
-  if (!(lanes == 0 || lanes == 1 || lanes == 2 || lanes == 4 || lanes == 8))
-    return fail(MLT_EINVAL, "lanes must be 0, 1, 2, 4 or 8");
-  if (!(group == 0 || group == 4 || group == 8)) return fail(MLT_EINVAL, "group must be 0, 4 or 8");
-  if (candidates && lanes && candidates * lanes > 256)
-    return fail(MLT_EINVAL, "candidates x lanes must be at most 256");
-  std::lock_guard<std::mutex> lk(g_mu);
-  g_shape[model_id].threads = candidates;
-  g_shape[model_id].lanes = lanes;
-  g_shape[model_id].group = group;
+  ShapeOverride& o = g_shape[model_id];
+  o.threads = candidates;
+  o.lanes = splits;
+  o.group = group;
+  o.chunk_trees = chunk_trees;
+  o.nbuf = nbuf;
   return MLT_OK;
 }
 

@@ -204,6 +204,20 @@ struct ShapeOverride {
   int group = 0;
 };
 
+// Full-table walk kernels for Q tree groups (Q = 1, 2 or 4), G in {2, 4, 8}
+// trees in flight, depth 1..10: traverse.cu / traverse_dec.cu (Q = 1),
+// traverse_q2.cu (Q = 2), traverse_q4.cu (Q = 4).  nullptr if not built.
+using FullKernelPtr = void (*)(TraverseArgs);
+using FullDecKernelPtr = void (*)(TraverseArgs, DecodeParams);
+FullKernelPtr full_kernel(int depth, int group, int q);
+FullDecKernelPtr full_dec_kernel(int depth, int group, int q);
+FullKernelPtr full_kernel_q1(int depth, int group);
+FullDecKernelPtr full_dec_kernel_q1(int depth, int group);
+FullKernelPtr full_kernel_q2(int depth, int group);
+FullDecKernelPtr full_dec_kernel_q2(int depth, int group);
+FullKernelPtr full_kernel_q4(int depth, int group);
+FullDecKernelPtr full_dec_kernel_q4(int depth, int group);
+
 // traverse.cu
 // n_eff: candidates the pass is expected to walk (used for load balance).
 ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, int sms,

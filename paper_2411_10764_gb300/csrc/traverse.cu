@@ -15,26 +15,18 @@ constexpr size_t kSmPerSm = 228 * 1024;  // shared memory per SM
 constexpr size_t kCtaReserve = 1024;     // reserved per resident CTA
 constexpr size_t kStaticSmem = 512;      // finish_tile and scan_tiles statics
 
-using FullKernel = void (*)(TraverseArgs);
+}  // namespace
 
-template <int G>
-FullKernel full_kernel(int d) {
-  switch (d) {
-    case 1: return k_traverse_full<1, G>;
-    case 2: return k_traverse_full<2, G>;
-    case 3: return k_traverse_full<3, G>;
-    case 4: return k_traverse_full<4, G>;
-    case 5: return k_traverse_full<5, G>;
-    case 6: return k_traverse_full<6, G>;
-    case 7: return k_traverse_full<7, G>;
-    case 8: return k_traverse_full<8, G>;
-    case 9: return k_traverse_full<9, G>;
-    case 10: return k_traverse_full<10, G>;
+FullKernelPtr full_kernel_q1(int depth, int group) { return full_kernel_q<1>(depth, group); }
+
+FullKernelPtr full_kernel(int depth, int group, int q) {
+  switch (q) {
+    case 1: return full_kernel_q1(depth, group);
+    case 2: return full_kernel_q2(depth, group);
+    case 4: return full_kernel_q4(depth, group);
     default: return nullptr;
   }
 }
-
-}  // namespace
 
 // Choose candidates per CTA (threads), trees per shared-memory chunk, chunk
 // buffers and trees walked together (group) for a full table.  Rules (from
@@ -48,25 +40,32 @@ FullKernel full_kernel(int d) {
 //     one CTA with bigger chunks: take the largest chunk that still allows
 //     two; otherwise one CTA with the largest chunk (fewest barriers);
 //   * a thread walks 8 trees at once when 8 warps or fewer share the SM,
-//     else 4 (the chunk permitting).
+//     else 4 (the chunk permitting);
+//   * a batch of under 32 (64) candidates per SM splits each tile's trees
+//     over 4 (2) groups of warps.
 ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms, int optin,
                       const ShapeOverride& ov) {
   if (sms < 1) sms = 1;
   if (n_eff < 1) n_eff = 1;
+  // tree groups per CTA: a batch of less than a warp (or two) per SM gets
+  // its trees split over 4 (2) groups of warps
+  const int q = ov.lanes ? ov.lanes : n_eff < 32LL * sms ? 4 : n_eff < 64LL * sms ? 2 : 1;
+  if (q != 1 && q != 2 && q != 4) return ScreenShape{};
   auto smem_of = [&](int tc, int chunk, int nb) {
-    return full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb);
+    return full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb, q, chunk);
   };
   auto fits = [&](size_t smem) { return smem + kStaticSmem <= static_cast<size_t>(optin); };
   auto resident = [&](size_t smem, int tc) {
     return static_cast<int>(std::min<size_t>(
-        {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / tc), 32}));
+        {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / (tc * q)), 32}));
   };
-  int tc = 256;
+  int tc = 256 / q;
   if (!ov.threads) {
     while (tc > 32 && (n_eff + tc - 1) / tc < (sms + 3) / 4) tc >>= 1;
   } else {
     tc = ov.threads;
   }
+  if (tc * q > 256) return ScreenShape{};
   const long long tiles = (n_eff + tc - 1) / tc;
   const long long tiles_sm = (tiles + sms - 1) / sms;
   ScreenShape best{};
@@ -85,10 +84,14 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
       const int rank = want2 * 1000 + chunk * 10 + (3 - nb);
       if (rank > best_rank) {
         best_rank = rank;
-        const int warps = res * tc / 32;
+        const int warps = res * tc * q / 32;
         int group = warps <= 8 ? 8 : 4;
-        group = std::min(group, chunk >= 8 ? 8 : chunk >= 4 ? 4 : 2);
+        if (ov.group) group = ov.group;
+        // each group walks chunk / q trees of a chunk
+        const int per = std::max(1, chunk / q);
+        group = std::min(group, per >= 8 ? 8 : per >= 4 ? 4 : 2);
         best.threads = tc;
+        best.lanes = q;
         best.chunk_trees = chunk;
         best.nbuf = nb;
         best.group = group;
@@ -109,7 +112,8 @@ ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes,
   if (tc < 64 || tc == s.threads) return s;
   ScreenShape b = s;
   b.threads = tc;
-  b.smem = full_smem_bytes(F, tc, s.nbuf, static_cast<uint32_t>(s.chunk_trees) * tree_bytes);
+  b.smem = full_smem_bytes(F, tc, s.nbuf, static_cast<uint32_t>(s.chunk_trees) * tree_bytes, s.lanes,
+                           s.chunk_trees);
   return b;
 }
 
@@ -134,8 +138,8 @@ ScreenShape plan_compact(int F, long long n_eff, int sms, int optin, const Shape
   if (n_eff < 1) n_eff = 1;
   for (int q : {1, 2, 4, 8}) {
     if (ov.lanes && q != ov.lanes) continue;
-    for (int tc : {256, 128, 64, 32}) {
-      if (ov.threads && tc != ov.threads) continue;
+    for (int tc : {256, 128, 64, 32, ov.threads}) {
+      if (tc == 0 || (ov.threads && tc != ov.threads)) continue;
       const int threads = tc * q;
       if (threads > 256) continue;
       const size_t smem = compact_smem_bytes(F, tc);
@@ -200,16 +204,14 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
     a.p_wave = shape.p_grid;
     ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
   }
-  const dim3 grid(static_cast<unsigned>(ctas)), block(shape.threads);
+  const dim3 grid(static_cast<unsigned>(ctas));
   if (m.kind == kTableFull) {
-    FullKernel k = shape.group == 8   ? full_kernel<8>(m.depth)
-                   : shape.group == 4 ? full_kernel<4>(m.depth)
-                                      : full_kernel<2>(m.depth);
+    FullKernelPtr k = full_kernel(m.depth, shape.group, shape.lanes);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, block, shape.smem, st, a);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, a);
     if (e != cudaSuccess) return e;
   } else {
     CompactKernel k = compact_kernel(shape.group, shape.lanes);

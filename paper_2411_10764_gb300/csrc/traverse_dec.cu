@@ -13,25 +13,6 @@ namespace {
 
 using namespace walk;
 
-using FullDecKernel = void (*)(TraverseArgs, DecodeParams);
-
-template <int G>
-FullDecKernel full_dec_kernel(int d) {
-  switch (d) {
-    case 1: return k_traverse_full_dec<1, G>;
-    case 2: return k_traverse_full_dec<2, G>;
-    case 3: return k_traverse_full_dec<3, G>;
-    case 4: return k_traverse_full_dec<4, G>;
-    case 5: return k_traverse_full_dec<5, G>;
-    case 6: return k_traverse_full_dec<6, G>;
-    case 7: return k_traverse_full_dec<7, G>;
-    case 8: return k_traverse_full_dec<8, G>;
-    case 9: return k_traverse_full_dec<9, G>;
-    case 10: return k_traverse_full_dec<10, G>;
-    default: return nullptr;
-  }
-}
-
 using CompactDecKernel = void (*)(TraverseArgs, DecodeParams);
 
 CompactDecKernel compact_dec_kernel(int group, int lanes) {
@@ -86,6 +67,17 @@ __global__ void __launch_bounds__(256)
 
 }  // namespace
 
+FullDecKernelPtr full_dec_kernel_q1(int depth, int group) { return full_dec_kernel_q<1>(depth, group); }
+
+FullDecKernelPtr full_dec_kernel(int depth, int group, int q) {
+  switch (q) {
+    case 1: return full_dec_kernel_q1(depth, group);
+    case 2: return full_dec_kernel_q2(depth, group);
+    case 4: return full_dec_kernel_q4(depth, group);
+    default: return nullptr;
+  }
+}
+
 cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, const DecodeParams& dec,
                                 const ScreenShape& shape, long long n_tiles, cudaStream_t st) {
   if (n_tiles <= 0) return cudaSuccess;
@@ -97,16 +89,14 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
     a.p_wave = shape.p_grid;
     ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
   }
-  const dim3 grid(static_cast<unsigned>(ctas)), block(shape.threads);
+  const dim3 grid(static_cast<unsigned>(ctas));
   if (m.kind == kTableFull) {
-    FullDecKernel k = shape.group == 8   ? full_dec_kernel<8>(m.depth)
-                      : shape.group == 4 ? full_dec_kernel<4>(m.depth)
-                                         : full_dec_kernel<2>(m.depth);
+    FullDecKernelPtr k = full_dec_kernel(m.depth, shape.group, shape.lanes);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k, grid, block, shape.smem, st, a, dec);
+    e = launch_pdl(k, grid, dim3(shape.threads * shape.lanes), shape.smem, st, a, dec);
     if (e != cudaSuccess) return e;
   } else {
     CompactDecKernel k = compact_dec_kernel(shape.group, shape.lanes);

@@ -363,24 +363,30 @@ __device__ __forceinline__ uint32_t go_right(float x, uint32_t thr_bits, uint32_
   return right;
 }
 
-// Walk trees [0, nt) of the chunk at shared address tb; xa = shared address
-// of this thread's feature column (feature f at xa + f * row_bytes).  The
-// 32-bit product meta * row_bytes drops meta's bit 31 because row_bytes is a
-// multiple of 2.
-template <int D, int G, bool NANP>
-__device__ __forceinline__ float walk_chunk(uint32_t tb, int nt, uint32_t tree_bytes, uint32_t xa,
-                                            uint32_t row_bytes, float acc) {
+__device__ __forceinline__ void sts_f32(uint32_t a, float v) {
+  asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(v) : "memory");
+}
+
+// Walk trees q, q + Q, q + 2Q, ... (< nt) of the chunk at shared address tb;
+// xa = shared address of this thread's feature column (feature f at xa + f *
+// row_bytes).  Q == 1: the leaves are added to acc in tree order.  Q > 1:
+// leaf t is parked at la + t * row_bytes for an in-order sum afterwards.
+// The 32-bit product meta * row_bytes drops meta's bit 31 because row_bytes
+// is a multiple of 2.
+template <int D, int G, bool NANP, int Q>
+__device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t tree_bytes, uint32_t xa,
+                                            uint32_t row_bytes, float acc, uint32_t la) {
   constexpr FullLayout L = full_layout(D);
   // byte offsets folded with the heap index of each region's first node
   constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
   constexpr uint32_t kMeta = L.off_meta - L.n_top * 4u;
   constexpr uint32_t kLast = L.off_last - L.n_inner * 16u;
-  int t = 0;
-  for (; t + G <= nt; t += G) {
+  int t = q;
+  for (; t + (G - 1) * Q < nt; t += G * Q) {
     uint32_t base[G], j[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      base[g] = tb + static_cast<uint32_t>(t + g) * tree_bytes;
+      base[g] = tb + static_cast<uint32_t>(t + g * Q) * tree_bytes;
       j[g] = 0;
     }
 #pragma unroll
@@ -412,10 +418,15 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int nt, uint32_t tree_b
 #pragma unroll
     for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
 #pragma unroll
-    for (int g = 0; g < G; ++g)
-      acc += __uint_as_float(go_right<NANP>(x[g], r[g].x, r[g].y) ? r[g].w : r[g].z);
+    for (int g = 0; g < G; ++g) {
+      const float leaf = __uint_as_float(go_right<NANP>(x[g], r[g].x, r[g].y) ? r[g].w : r[g].z);
+      if (Q == 1)
+        acc += leaf;
+      else
+        sts_f32(la + static_cast<uint32_t>(t + g * Q) * row_bytes, leaf);
+    }
   }
-  for (; t < nt; ++t) {
+  for (; t < nt; t += Q) {
     const uint32_t base = tb + static_cast<uint32_t>(t) * tree_bytes;
     uint32_t j = 0;
 #pragma unroll
@@ -434,21 +445,33 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int nt, uint32_t tree_b
     }
     const uint4 r = lds_u4(base + kLast + j * 16u);
     const float x = lds_f32(r.y * row_bytes + xa);
-    acc += __uint_as_float(go_right<NANP>(x, r.x, r.y) ? r.w : r.z);
+    const float leaf = __uint_as_float(go_right<NANP>(x, r.x, r.y) ? r.w : r.z);
+    if (Q == 1)
+      acc += leaf;
+    else
+      sts_f32(la + static_cast<uint32_t>(t) * row_bytes, leaf);
   }
   return acc;
 }
 
 // Shared-memory layout of the full-table kernel (host and device agree):
-//   [0, feat) features [F][TC]; rows [TC] u32; nbuf chunk buffers; mbarriers.
+//   features [F][TC]; rows [TC] u32; nbuf chunk buffers; with Q > 1 tree
+//   groups, two parked-leaf buffers [chunk_trees][TC] fp32; mbarriers.
 __host__ __device__ inline size_t full_smem_rows_off(int F, int TC) {
   return align_up(static_cast<size_t>(F) * TC * 4, 128);
 }
 __host__ __device__ inline size_t full_smem_tbuf_off(int F, int TC) {
   return full_smem_rows_off(F, TC) + align_up(static_cast<size_t>(TC) * 4, 128);
 }
-__host__ __device__ inline size_t full_smem_bytes(int F, int TC, int nbuf, uint32_t chunk_bytes) {
-  return align_up(full_smem_tbuf_off(F, TC) + static_cast<size_t>(nbuf) * chunk_bytes, 16) + 8 * 4;
+__host__ __device__ inline size_t full_smem_leaf_off(int F, int TC, int nbuf, uint32_t chunk_bytes) {
+  return align_up(full_smem_tbuf_off(F, TC) + static_cast<size_t>(nbuf) * chunk_bytes, 16);
+}
+__host__ __device__ inline size_t full_smem_leaf_bytes(int TC, int Q, int chunk_trees) {
+  return Q > 1 ? 2 * static_cast<size_t>(chunk_trees) * TC * 4 : 0;
+}
+__host__ __device__ inline size_t full_smem_bytes(int F, int TC, int nbuf, uint32_t chunk_bytes, int Q,
+                                                  int chunk_trees) {
+  return full_smem_leaf_off(F, TC, nbuf, chunk_bytes) + full_smem_leaf_bytes(TC, Q, chunk_trees) + 8 * 4;
 }
 
 // Even split of `len` items into `parts` contiguous pieces whose sizes
@@ -486,27 +509,38 @@ __device__ __forceinline__ void cta_tile(const TraverseArgs& a, long long count,
   *len = static_cast<int>(split_start(S, tiles, blockIdx.x + 1) - lo);
 }
 
-template <int D, int G>
+// Full-table walk of one tile.  The CTA has Q groups of TC threads (TC =
+// candidates of the tile, a multiple of 32).  Thread c of group q walks
+// trees q, q + Q, ... of every chunk for candidate c; with Q > 1 it parks
+// the leaves in shared memory and group 0 adds each chunk's leaves in tree
+// order one chunk later (two leaf buffers), so the sum is the same
+// sequential fp32 sum as with one walker.  More groups put more warps on a
+// small batch; all lanes of a warp still walk the same tree.
+template <int D, int G, int Q>
 __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
   extern __shared__ __align__(128) unsigned char smem[];
-  const int TC = blockDim.x;
+  const int TC = blockDim.x / Q;
   const int tid = threadIdx.x;
-  const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
+  const int q = Q == 1 ? 0 : tid / TC;  // warp-uniform (TC is a multiple of 32)
+  const int c = Q == 1 ? tid : tid - q * TC;
   // the P pass needs the survivor count of the kernels before it; the V
   // pass only needs them before it reads the features, unless a batched call
   // must first learn whether an earlier batch already reached its target
   if (a.p_pass || a.stream) pdl_wait();
   if (a.stream && *reinterpret_cast<volatile const unsigned*>(&a.stream->done)) return;
   const long long count = a.p_pass ? static_cast<long long>(a.state->survivors) : a.n;
-  if (tile0 >= count) return;  // whole CTA, before any copy is issued
-  const int rows_here = static_cast<int>(min(static_cast<long long>(TC), count - tile0));
+  long long tile0;
+  int rows_here;
+  cta_tile(a, count, TC, &tile0, &rows_here);
+  if (rows_here <= 0) return;  // whole CTA, before any copy is issued
 
   float* xs = reinterpret_cast<float*>(smem);
   uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + full_smem_rows_off(a.F, TC));
   unsigned char* tbuf = smem + full_smem_tbuf_off(a.F, TC);
   const uint32_t chunk_bytes = static_cast<uint32_t>(a.chunk_trees) * a.tree_bytes;
+  const size_t leaf_off = full_smem_leaf_off(a.F, TC, a.nbuf, chunk_bytes);
   unsigned long long* bars = reinterpret_cast<unsigned long long*>(
-      smem + align_up(full_smem_tbuf_off(a.F, TC) + static_cast<size_t>(a.nbuf) * chunk_bytes, 16));
+      smem + leaf_off + full_smem_leaf_bytes(TC, Q, a.chunk_trees));
   const int n_chunks = (a.n_trees + a.chunk_trees - 1) / a.chunk_trees;
 
   if (tid == 0) {
@@ -514,8 +548,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     fence_mbar_init();
   }
   __syncthreads();
-  auto issue = [&](int c, int b) {
-    const int first = c * a.chunk_trees;
+  auto issue = [&](int ch, int b) {
+    const int first = ch * a.chunk_trees;
     const int nt = min(a.chunk_trees, a.n_trees - first);
     const uint32_t bytes = static_cast<uint32_t>(nt) * a.tree_bytes;
     const uint32_t bar = smem_u32(&bars[b]);
@@ -524,51 +558,120 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
                   a.table + static_cast<size_t>(first) * a.tree_bytes, bytes, bar);
   };
   if (tid == 0)
-    for (int c = 0; c < a.nbuf && c < n_chunks; ++c) issue(c, c);  // tables are static
+    for (int ch = 0; ch < a.nbuf && ch < n_chunks; ++ch) issue(ch, ch);  // tables are static
 
   if (!a.p_pass) pdl_wait();
   if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
-  // each thread stages its own row (and reads only its own rowidx entry)
-  const bool nan = __syncthreads_or(stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+  // group 0 stages one row per thread (a thread reads only its own rowidx
+  // entry); every group reads the same feature columns
+  const bool nan = __syncthreads_or(tid < TC && stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+  // warps past the tile's rows walk zero features: a branch around their
+  // walk measured slower than the idle work (it changes the code of the
+  // walk loop)
+  const bool live = (c & ~31) < rows_here;
 
   float acc = 0.0f;
   const uint32_t row_bytes = static_cast<uint32_t>(TC) * 4u;
-  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(tid) * 4u;
+  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(c) * 4u;
   const uint32_t tbuf_a = smem_u32(tbuf);
-  for (int c = 0; c < n_chunks; ++c) {
-    const int b = c % a.nbuf;
-    const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(c / a.nbuf) & 1u);
+  // parked leaves: buffer p holds leaf t of candidate c at la[p] + t * row_bytes
+  const uint32_t la0 = smem_u32(smem + leaf_off) + static_cast<uint32_t>(c) * 4u;
+  const uint32_t la_step = static_cast<uint32_t>(a.chunk_trees) * row_bytes;
+  for (int ch = 0; ch < n_chunks; ++ch) {
+    const int b = ch % a.nbuf;
+    const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
     if (!__syncthreads_and(ok)) {
       if (tid == 0) {
         // let every copy still in flight land before the CTA's shared memory
         // is released, then report
-        for (int cc = c + 1; cc < n_chunks && cc < c + a.nbuf; ++cc)
+        for (int cc = ch + 1; cc < n_chunks && cc < ch + a.nbuf; ++cc)
           mbar_wait_bounded(smem_u32(&bars[cc % a.nbuf]), static_cast<uint32_t>(cc / a.nbuf) & 1u);
-        mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(c / a.nbuf) & 1u);
+        mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
         atomicOr(a.err, kErrWaitTimeout);
       }
       return;
     }
     const uint32_t tb = tbuf_a + static_cast<uint32_t>(b) * chunk_bytes;
-    const int nt = min(a.chunk_trees, a.n_trees - c * a.chunk_trees);
-    acc = nan ? walk_chunk<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
-              : walk_chunk<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+    const int nt = min(a.chunk_trees, a.n_trees - ch * a.chunk_trees);
+    const uint32_t la = la0 + static_cast<uint32_t>(ch & 1) * la_step;
+    acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
+              : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);
+    if (Q > 1 && q == 0 && ch > 0) {
+      // the previous chunk's leaves (complete since the last barrier)
+      const uint32_t lp = la0 + static_cast<uint32_t>((ch - 1) & 1) * la_step;
+      const int np = live ? a.chunk_trees : 0;  // every chunk but the last is full
+      for (int t = 0; t < np; ++t) acc += lds_f32(lp + static_cast<uint32_t>(t) * row_bytes);
+    }
     __syncthreads();
-    if (tid == 0 && c + a.nbuf < n_chunks) issue(c + a.nbuf, b);
+    if (tid == 0 && ch + a.nbuf < n_chunks) issue(ch + a.nbuf, b);
+  }
+  if (Q > 1 && q == 0) {
+    const uint32_t lp = la0 + static_cast<uint32_t>((n_chunks - 1) & 1) * la_step;
+    const int np = live ? a.n_trees - (n_chunks - 1) * a.chunk_trees : 0;
+    for (int t = 0; t < np; ++t) acc += lds_f32(lp + static_cast<uint32_t>(t) * row_bytes);
   }
   pdl_trigger();
   finish_tile(a, rowidx, tile0, rows_here, count, acc, TC);
 }
 
-template <int D, int G>
+template <int D, int G, int Q>
 __global__ void __launch_bounds__(256) k_traverse_full(const __grid_constant__ TraverseArgs a) {
-  traverse_full_body<D, G>(a, nullptr);
+  traverse_full_body<D, G, Q>(a, nullptr);
 }
 
-template <int D, int G>
+template <int D, int G, int Q>
 __global__ void __launch_bounds__(256)
     k_traverse_full_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
-  traverse_full_body<D, G>(a, &d);
+  traverse_full_body<D, G, Q>(a, &d);
+}
+
+// Kernel of depth d (1..10) for G trees in flight and Q tree groups.
+template <int G, int Q>
+FullKernelPtr full_kernel_for(int d) {
+  switch (d) {
+    case 1: return k_traverse_full<1, G, Q>;
+    case 2: return k_traverse_full<2, G, Q>;
+    case 3: return k_traverse_full<3, G, Q>;
+    case 4: return k_traverse_full<4, G, Q>;
+    case 5: return k_traverse_full<5, G, Q>;
+    case 6: return k_traverse_full<6, G, Q>;
+    case 7: return k_traverse_full<7, G, Q>;
+    case 8: return k_traverse_full<8, G, Q>;
+    case 9: return k_traverse_full<9, G, Q>;
+    case 10: return k_traverse_full<10, G, Q>;
+    default: return nullptr;
+  }
+}
+
+template <int G, int Q>
+FullDecKernelPtr full_dec_kernel_for(int d) {
+  switch (d) {
+    case 1: return k_traverse_full_dec<1, G, Q>;
+    case 2: return k_traverse_full_dec<2, G, Q>;
+    case 3: return k_traverse_full_dec<3, G, Q>;
+    case 4: return k_traverse_full_dec<4, G, Q>;
+    case 5: return k_traverse_full_dec<5, G, Q>;
+    case 6: return k_traverse_full_dec<6, G, Q>;
+    case 7: return k_traverse_full_dec<7, G, Q>;
+    case 8: return k_traverse_full_dec<8, G, Q>;
+    case 9: return k_traverse_full_dec<9, G, Q>;
+    case 10: return k_traverse_full_dec<10, G, Q>;
+    default: return nullptr;
+  }
+}
+
+// All depths and G in {2, 4, 8} for one Q (each Q is instantiated in its own
+// translation unit, compiled in parallel).
+template <int Q>
+FullKernelPtr full_kernel_q(int d, int g) {
+  return g == 8 ? full_kernel_for<8, Q>(d) : g == 4 ? full_kernel_for<4, Q>(d) : g == 2 ? full_kernel_for<2, Q>(d) : nullptr;
+}
+template <int Q>
+FullDecKernelPtr full_dec_kernel_q(int d, int g) {
+  return g == 8   ? full_dec_kernel_for<8, Q>(d)
+         : g == 4 ? full_dec_kernel_for<4, Q>(d)
+         : g == 2 ? full_dec_kernel_for<2, Q>(d)
+                  : nullptr;
 }
 
 // ---------------------------------------------------------------------------

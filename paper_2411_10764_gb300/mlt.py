@@ -67,8 +67,7 @@ def lib(build_if_missing: bool = True):
             "mlt_last_survivor_count": [P, P],
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
-            "mlt_tune_shape": [i32, i32, i32, i32],
-            "mlt_tune_deep_walk": [i32, i32, i32, i32],
+            "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
             "mlt_screen_until": [P, P, i64, i64, i64, f32, i32, P, P, P, P],
@@ -324,14 +323,11 @@ def phase_times():
     return dict(zip(PHASES, [float(v) for v in out])), int(calls.value)
 
 
-def tune_shape(model_id: int, threads: int = 0, chunk_trees: int = 0, nbuf: int = 0) -> None:
-    """Fix (or with zeros, release) the walk's launch shape for one model."""
-    _check(lib().mlt_tune_shape(int(model_id), int(threads), int(chunk_trees), int(nbuf)))
-
-
-def tune_deep_walk(model_id: int, candidates: int = 0, lanes: int = 0, group: int = 0) -> None:
-    """Fix (or with zeros, release) the deep-tree walk's launch shape for one model."""
-    _check(lib().mlt_tune_deep_walk(int(model_id), int(candidates), int(lanes), int(group)))
+def tune_walk(model_id: int, candidates: int = 0, splits: int = 0, group: int = 0, chunk_trees: int = 0,
+              nbuf: int = 0) -> None:
+    """Fix (or with zeros, release) the tree walk's launch shape for one model."""
+    _check(lib().mlt_tune_walk(int(model_id), int(candidates), int(splits), int(group), int(chunk_trees),
+                               int(nbuf)))
 
 
 def kernel_launches() -> int:

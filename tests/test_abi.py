@@ -131,16 +131,15 @@ def test_decoder_validation(L):
     assert call(r, prog, 0, 1, F=257) == -1
 
 
-@pytest.mark.parametrize("args", [(0, 48, 1, 4), (0, 64, 3, 4), (0, 64, 8, 4), (0, 64, 4, 2), (5, 64, 4, 4)])
-def test_deep_walk_tuning_rejects(args):
-    from paper_2411_10764_gb300 import mlt
-
+@pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 64, 8, 4, 0, 0),
+                                  (0, 64, 4, 3, 0, 0), (5, 64, 4, 4, 0, 0), (0, 0, 0, 0, 3, 0),
+                                  (0, 0, 0, 0, 0, 4), (0, 288, 1, 4, 0, 0)])
+def test_walk_tuning_rejects(args):
     with pytest.raises(mlt.MltError):
-        mlt.tune_deep_walk(*args)
+        mlt.tune_walk(*args)
 
 
-def test_deep_walk_tuning_accepts_and_releases():
-    from paper_2411_10764_gb300 import mlt
-
-    mlt.tune_deep_walk(mlt.MLT_MODEL_P, 64, 4, 8)
-    mlt.tune_deep_walk(mlt.MLT_MODEL_P)
+def test_walk_tuning_accepts_and_releases():
+    mlt.tune_walk(mlt.MLT_MODEL_P, 64, 4, 8, 8, 2)
+    mlt.tune_walk(mlt.MLT_MODEL_P, 96, 2, 2, 16, 3)
+    mlt.tune_walk(mlt.MLT_MODEL_P)

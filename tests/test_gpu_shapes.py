@@ -46,8 +46,12 @@ def full():
 
 def _release():
     for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
-        mlt.tune_shape(m)
-        mlt.tune_deep_walk(m)
+        mlt.tune_walk(m)
+
+
+def _force(**shape):
+    for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
+        mlt.tune_walk(m, **shape)
 
 
 DEEP_SHAPES = [(c, q, g) for c in (32, 64, 128, 256) for q in (1, 2, 4, 8) for g in (4, 8) if c * q <= 256]
@@ -56,8 +60,7 @@ DEEP_SHAPES = [(c, q, g) for c in (32, 64, 128, 256) for q in (1, 2, 4, 8) for g
 @pytest.mark.parametrize("cand,lanes,group", DEEP_SHAPES)
 def test_deep_walk_every_shape(deep, cand, lanes, group):
     try:
-        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
-            mlt.tune_deep_walk(m, cand, lanes, group)
+        _force(candidates=cand, splits=lanes, group=group)
         got = gpu_screen(deep)
     finally:
         _release()
@@ -67,8 +70,7 @@ def test_deep_walk_every_shape(deep, cand, lanes, group):
 @pytest.mark.parametrize("cand,lanes,group", [(32, 8, 4), (64, 4, 8), (128, 1, 8), (32, 2, 8)])
 def test_deep_walk_decoded_shapes(deep_decoded, cand, lanes, group):
     try:
-        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
-            mlt.tune_deep_walk(m, cand, lanes, group)
+        _force(candidates=cand, splits=lanes, group=group)
         got = gpu_screen(deep_decoded)
     finally:
         _release()
@@ -81,9 +83,48 @@ FULL_SHAPES = [(t, c, b) for t in (32, 64, 128, 256) for c in (1, 2, 4, 8, 16) f
 @pytest.mark.parametrize("threads,chunk,nbuf", FULL_SHAPES)
 def test_full_walk_every_shape(full, threads, chunk, nbuf):
     try:
-        for m in (mlt.MLT_MODEL_V, mlt.MLT_MODEL_P):
-            mlt.tune_shape(m, threads, chunk, nbuf)
+        _force(candidates=threads, chunk_trees=chunk, nbuf=nbuf)
         got = gpu_screen(full)
     finally:
         _release()
     assert_parity(got, _expected("full", full))
+
+
+# tree groups: warps of a CTA split each chunk's trees, leaves summed in order
+SPLIT_SHAPES = ([(t, 2, g, c) for t in (32, 64, 96, 128) for c in (1, 4, 16) for g in (2, 4, 8)] +
+                [(t, 4, g, c) for t in (32, 64) for c in (2, 8, 16) for g in (4, 8)])
+
+
+@pytest.mark.parametrize("cand,splits,group,chunk", SPLIT_SHAPES)
+def test_full_walk_tree_groups(full, cand, splits, group, chunk):
+    try:
+        _force(candidates=cand, splits=splits, group=group, chunk_trees=chunk, nbuf=2)
+        got = gpu_screen(full)
+    finally:
+        _release()
+    assert_parity(got, _expected("full", full))
+
+
+@pytest.mark.parametrize("cand", [96, 160, 224])
+def test_full_walk_candidate_counts_not_powers_of_two(full, cand):
+    try:
+        _force(candidates=cand)
+        got = gpu_screen(full)
+    finally:
+        _release()
+    assert_parity(got, _expected("full", full))
+
+
+@pytest.fixture(scope="module")
+def decoded():
+    return W.make_workload(4, seed=3, n=7001)
+
+
+@pytest.mark.parametrize("cand,splits,group,chunk", [(128, 2, 8, 16), (64, 4, 4, 8), (96, 2, 4, 4), (256, 1, 8, 4)])
+def test_full_walk_decoded_shapes(decoded, cand, splits, group, chunk):
+    try:
+        _force(candidates=cand, splits=splits, group=group, chunk_trees=chunk, nbuf=2)
+        got = gpu_screen(decoded)
+    finally:
+        _release()
+    assert_parity(got, _expected("decoded", decoded))
