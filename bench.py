@@ -422,6 +422,47 @@ def run_ours(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
 
+    # the half-table variant (binary16 thresholds, leaves and staged
+    # features): same batch, same timing protocol; it changes results, so
+    # its agreement with the fp32 run is reported beside its speed
+    half = None
+    if not args.no_half and d is None and max(w.v.depth, w.p.depth) <= 10:
+        ref_valid = torch.isfinite(pf).cpu().numpy()
+        ref_topk = tk.cpu().numpy()
+        mlt.load_workload_models(w, half=True)
+        for _ in range(max(3, args.warmup)):
+            flush.fill_(1.0)
+            step()
+        h_steps = max(10, min(args.steps, 500))
+        hs = [torch.cuda.Event(enable_timing=True) for _ in range(h_steps)]
+        he = [torch.cuda.Event(enable_timing=True) for _ in range(h_steps)]
+        torch.cuda.synchronize(dev)
+        for i in range(h_steps):
+            flush.fill_(float(i))
+            hs[i].record(stream)
+            step()
+            he[i].record(stream)
+        torch.cuda.synchronize(dev)
+        mlt.sync_status(stream)
+        h_ms = float(sum(a.elapsed_time(b) for a, b in zip(hs, he))) / h_steps
+        mlt.profile_phases(True)
+        for i in range(min(h_steps, 50)):
+            flush.fill_(float(i))
+            step()
+        h_phases, h_calls = mlt.phase_times()
+        mlt.profile_phases(False)
+        h_valid = torch.isfinite(pf).cpu().numpy()
+        h_topk = tk.cpu().numpy()
+        half = {"value": world * n / (h_ms / 1e3), "unit": "candidates/s", "ms_per_step": h_ms,
+                "steps": h_steps,
+                "phases_ms": {kk: vv / max(h_calls, 1) for kk, vv in h_phases.items()},
+                "decision_agreement": float((h_valid == ref_valid).mean()),
+                "topk_overlap": len(set(h_topk.tolist()) & set(ref_topk.tolist())) / k,
+                "what": "mlt_load_ensemble_f16: binary16 thresholds, leaves and staged features; "
+                        "changes results (parity is against the rounded model); agreement and top-k "
+                        "overlap are against the fp32 run on the same batch"}
+        mlt.load_workload_models(w)
+
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
@@ -471,6 +512,7 @@ def run_ours(args):
                 "d2h_bytes_per_step": int(2 * n * 4 + k * 8)},
         "gpu_launches": int(launches),
         "rerank": rerank,
+        "half_tables": half,
         "clocks": clocks,
         "wall_ms_per_step_incl_flush": wall * 1e3 / args.steps,
     }
@@ -496,6 +538,7 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-rerank", action="store_true")
+    ap.add_argument("--no-half", action="store_true", help="skip the half-table variant's timing")
     ap.add_argument("--n", type=int, default=None,
                     help="candidates per batch (default: the workload's size; smaller for profiling captures)")
     args = ap.parse_args()

@@ -111,6 +111,21 @@ int mlt_set_num_features(int F);
  * Synchronous (waits for queued work before freeing an old table). */
 int mlt_load_ensemble(int model_id, const mlt_node *nodes, int n_trees, int depth);
 
+/* Half tables: like mlt_load_ensemble, but the ensemble is stored with its
+ * thresholds and leaves rounded to IEEE binary16 (round to nearest even),
+ * and every screening pass over this model rounds the candidate's features
+ * to binary16 too.  Halves the table and the staged features, and changes
+ * results: the call screens exactly as the rounded model scores the rounded
+ * rows (comparisons in binary16, leaves summed in fp32 in tree order), so
+ * decisions and scores may differ from the fp32 model near split
+ * thresholds and by the rounding of the leaves.  For models V and P of
+ * depth 1 .. 10 with F <= 1024; a leaf whose magnitude rounds past 65504 is
+ * MLT_EINVAL (a threshold that does is kept as an infinity).  Screening
+ * calls that build features from candidate indices (mlt_screen_decoded,
+ * mlt_screen_until_decoded, mlt_sa_step) return MLT_EINVAL while a half
+ * table is loaded.  Synchronous. */
+int mlt_load_ensemble_f16(int model_id, const mlt_node *nodes, int n_trees, int depth);
+
 /* Free a loaded ensemble (no-op if the slot is empty).  Synchronous. */
 int mlt_free_ensemble(int model_id);
 

@@ -10,8 +10,10 @@ from .oracle import (  # noqa: F401
     build,
     decode,
     features,
+    half_ensemble,
     margins,
     rerank,
+    round_half,
     sa_step,
     screen,
     screen_rows,

@@ -300,3 +300,27 @@ def features(radices, option_values, program, first: int, n: int, threads: int =
     if any(s != 0 for s in status):
         raise ValueError("index beyond the knob space or malformed feature program")
     return knobs, feats
+
+
+# ---------------------------------------------------------------------------
+# Half tables (binary16 thresholds, leaves and features): the rounded model
+# ---------------------------------------------------------------------------
+def round_half(a) -> np.ndarray:
+    """IEEE 754 binary16 rounding of fp32 values (round to nearest, ties to
+    even; magnitudes from 65520 up become infinities; NaN stays NaN),
+    returned as fp32 -- exact, since every binary16 value is an fp32 value.
+    numpy's float16 conversion implements this rounding."""
+    with np.errstate(over="ignore"):
+        return np.asarray(a, dtype=np.float32).astype(np.float16).astype(np.float32)
+
+
+def half_ensemble(ensemble):
+    """The ensemble half tables hold: every split threshold and leaf value
+    rounded to binary16 (same shape and features).  Screening the rounded
+    rows (round_half) with it is the half-table variant's exact result."""
+    nodes, n_trees, depth = _ens(ensemble)
+    out = np.array(nodes, copy=True)
+    used = out["feature"] != -2
+    out["value"][used] = round_half(out["value"][used])
+    return (out, n_trees, depth)
+

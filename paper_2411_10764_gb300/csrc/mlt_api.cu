@@ -19,6 +19,8 @@
 #include <vector>
 
 #include "mlt.h"
+#include <cuda_fp16.h>
+
 #include "mlt_internal.cuh"
 
 // Scratch of mlt_screen_noalloc: one fixed array in the module's global
@@ -237,12 +239,16 @@ int check_screen_args(long long n, float thr, int k) {
   return MLT_OK;
 }
 
-int check_models(int dev) {
+// decoded: the features are built from candidate indices (half tables need
+// a stored feature matrix).
+int check_models(int dev, bool decoded = false) {
   for (int id : {MLT_MODEL_V, MLT_MODEL_P}) {
     const Model& m = g_models[id];
     if (!m.loaded) return fail(MLT_ENOMODEL, "model %s is not loaded", id == 0 ? "V" : "P");
     if (m.F != g_F) return fail(MLT_ENOMODEL, "model %s was loaded for F=%d, current F=%d", id == 0 ? "V" : "P", m.F, g_F);
     if (m.device != dev) return fail(MLT_EINVAL, "model %s lives on device %d, current device is %d", id == 0 ? "V" : "P", m.device, dev);
+    if (decoded && m.dm.kind == kTableHalf)
+      return fail(MLT_EINVAL, "model %s has half tables, which need stored features", id == 0 ? "V" : "P");
   }
   return MLT_OK;
 }
@@ -250,14 +256,17 @@ int check_models(int dev) {
 // v_pass: n_eff is the exact number of candidates; otherwise it is an
 // estimate of the survivors.  Full-table tiles are balanced over the SMs.
 ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov, bool v_pass) {
-  ScreenShape s = dm.kind == kTableFull
-                      ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
+  const bool half = dm.kind == kTableHalf;
+  ScreenShape s = dm.kind != kTableCompact
+                      ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov, half)
                       : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
   if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
     return plan_for(dm, F, n_eff, ShapeOverride(), v_pass);
   // the P pass splits its survivors evenly over the CTAs on the device, so
   // its CTA size is balanced for the estimate as well
-  if (dm.kind == kTableFull && ov.threads == 0) s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count());
+  if (dm.kind != kTableCompact && ov.threads == 0)
+    s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count(), half);
+  if (dm.kind != kTableCompact) s = cap_residency(s, smem_optin());
   return s;
 }
 
@@ -429,7 +438,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   int dev = 0;
   int rc = current_device(&dev);
   if (rc != MLT_OK) return rc;
-  rc = check_models(dev);
+  rc = check_models(dev, dec != nullptr);
   if (rc != MLT_OK) return rc;
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
@@ -539,7 +548,7 @@ int run_stream(cudaStream_t st, const float* feats, const DecodeParams* dec0, lo
   int dev = 0;
   int rc = current_device(&dev);
   if (rc != MLT_OK) return rc;
-  rc = check_models(dev);
+  rc = check_models(dev, dec0 != nullptr);
   if (rc != MLT_OK) return rc;
   rc = ensure_scratch(n_total);  // every kept survivor's key fits
   if (rc != MLT_OK) return rc;
@@ -637,6 +646,98 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   return run_screen_with(st, feats, dec, n, thr, k, out_pvalid, out_perf, out_topk, g_scr.s, true);
 }
 
+// Half table (kTableHalf): validate like pack_ensemble, then store the
+// complete heap with binary16 thresholds and leaves (round to nearest even).
+int pack_ensemble_half(const mlt_node* nodes, int n_trees, int depth, int F, std::vector<unsigned char>& out,
+                       DeviceModel& dm) {
+  {
+    std::vector<unsigned char> scratch;
+    DeviceModel probe;
+    const int rc = pack_ensemble(nodes, n_trees, depth, F, scratch, probe);  // validation
+    if (rc != MLT_OK) return rc;
+  }
+  const int slots = (2 << depth) - 1;
+  const HalfLayout lay = half_layout(depth);
+  const size_t tb = lay.bytes;
+  const int inner = (1 << depth) - 1;  // internal heap slots of the complete tree
+  dm.kind = kTableHalf;
+  dm.n_trees = n_trees;
+  dm.depth = depth;
+  dm.tree_bytes = lay.bytes;
+  out.assign(tb * n_trees, 0);
+  std::vector<unsigned char> reach(slots);
+  std::vector<float> inherit(slots);
+  std::vector<uint32_t> word(inner);
+  auto h16 = [](float v) { return static_cast<uint32_t>(__half_as_ushort(__float2half_rn(v))); };
+  for (int t = 0; t < n_trees; ++t) {
+    const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+    unsigned char* dst = out.data() + tb * t;
+    std::fill(reach.begin(), reach.end(), 0);
+    reach[0] = 1;
+    for (int j = 0; j < slots; ++j) {
+      const mlt_node& nd = tr[j];
+      const bool split = reach[j] && nd.feature >= 0;
+      if (split) {
+        reach[2 * j + 1] = 1;
+        reach[2 * j + 2] = 1;
+      }
+      if (reach[j] && nd.feature == -1) {
+        const uint32_t lb = h16(nd.value);
+        if ((lb & 0x7C00u) == 0x7C00u)
+          return fail(MLT_EINVAL, "tree %d slot %d: leaf %g does not fit binary16", t, j, nd.value);
+        inherit[j] = nd.value;
+      } else if (!reach[j]) {
+        inherit[j] = inherit[(j - 1) / 2];  // below a leaf: copy it down
+      } else {
+        inherit[j] = 0.0f;
+      }
+      if (j < inner)
+        word[j] = split ? (h16(nd.value) | (static_cast<uint32_t>(nd.feature) << kHalfFeatureShift) |
+                           (nd.default_left ? kMetaDefaultLeft : 0u))
+                        : 0u;  // pass-through: threshold 0 on feature 0, both sides lead to the same leaf
+    }
+    for (uint32_t j = 0; j < static_cast<uint32_t>(inner); ++j) {
+      if (j < lay.n_inner) {
+        std::memcpy(dst + 4 * j, &word[j], 4);
+      } else {
+        unsigned char* rec = dst + lay.off_last + 8 * (j - lay.n_inner);
+        const uint32_t leaves = h16(inherit[2 * j + 1]) | (h16(inherit[2 * j + 2]) << 16);
+        std::memcpy(rec, &word[j], 4);
+        std::memcpy(rec + 4, &leaves, 4);
+      }
+    }
+  }
+  return MLT_OK;
+}
+
+// Upload a packed table into model slot `model_id` (lock held).
+int install_model(int model_id, const std::vector<unsigned char>& packed, const DeviceModel& dm) {
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  unsigned char* d = nullptr;
+  cudaError_t e = cudaMalloc(&d, packed.size());
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(MLT_ENOMEM, "cannot allocate %zu bytes for the ensemble", packed.size());
+  }
+  e = cudaMemcpy(d, packed.data(), packed.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cudaFree(d);
+    return cuda_fail(e, "ensemble upload");
+  }
+  free_model(g_models[model_id]);
+  Model& m = g_models[model_id];
+  m.loaded = true;
+  m.device = dev;
+  m.F = g_F;
+  m.owned = d;
+  m.dm = dm;
+  m.dm.table = d;
+  m.dm.bytes = packed.size();
+  return MLT_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -661,30 +762,24 @@ int mlt_load_ensemble(int model_id, const mlt_node* nodes, int n_trees, int dept
   DeviceModel dm;
   int rc = pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
   if (rc != MLT_OK) return rc;
-  int dev = 0;
-  rc = current_device(&dev);
+  return install_model(model_id, packed, dm);
+}
+
+int mlt_load_ensemble_f16(int model_id, const mlt_node* nodes, int n_trees, int depth) {
+  if (model_id != MLT_MODEL_V && model_id != MLT_MODEL_P)
+    return fail(MLT_EINVAL, "half tables are for models V and P, got model id %d", model_id);
+  if (nodes == nullptr) return fail(MLT_EINVAL, "nodes must be non-NULL");
+  if (n_trees < 1 || n_trees > 65536) return fail(MLT_EINVAL, "n_trees must lie in [1, 65536], got %d", n_trees);
+  if (depth < 1 || depth > kMaxFullDepth)
+    return fail(MLT_EINVAL, "half tables need depth in [1, %d], got %d", kMaxFullDepth, depth);
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_EINVAL, "call mlt_set_num_features before loading ensembles");
+  if (g_F > static_cast<int>(kHalfFeatureMask) + 1) return fail(MLT_EINVAL, "half tables need F <= 1024");
+  std::vector<unsigned char> packed;
+  DeviceModel dm;
+  int rc = pack_ensemble_half(nodes, n_trees, depth, g_F, packed, dm);
   if (rc != MLT_OK) return rc;
-  unsigned char* d = nullptr;
-  cudaError_t e = cudaMalloc(&d, packed.size());
-  if (e != cudaSuccess) {
-    cudaGetLastError();
-    return fail(MLT_ENOMEM, "cannot allocate %zu bytes for the ensemble", packed.size());
-  }
-  e = cudaMemcpy(d, packed.data(), packed.size(), cudaMemcpyHostToDevice);
-  if (e != cudaSuccess) {
-    cudaFree(d);
-    return cuda_fail(e, "ensemble upload");
-  }
-  free_model(g_models[model_id]);
-  Model& m = g_models[model_id];
-  m.loaded = true;
-  m.device = dev;
-  m.F = g_F;
-  m.owned = d;
-  m.dm = dm;
-  m.dm.table = d;
-  m.dm.bytes = packed.size();
-  return MLT_OK;
+  return install_model(model_id, packed, dm);
 }
 
 int mlt_free_ensemble(int model_id) {

@@ -50,7 +50,33 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 //   meta bit 30 = leaf (value = leaf output), bit 31 = NaN goes left,
 //   bits 10..29 = index of the left child within the tree (right = left+1),
 //   bits 0..9 = feature index (F <= 1024).
-enum TableKind : int { kTableFull = 0, kTableCompact = 1 };
+//
+// Half table (depth D <= kMaxFullDepth, loaded by mlt_load_ensemble_f16):
+// the full table's heap with thresholds and leaves rounded to IEEE binary16
+// (round to nearest even), `tree_bytes` apart:
+//   levels [0, D-1)  : 4-byte words {bits 0..15 threshold (binary16), bits
+//                      16..25 feature index, bit 31 NaN goes left};
+//   level D-1 (last) : 8-byte records {that word; left leaf | right leaf << 16
+//                      (binary16)}.
+// The features are rounded to binary16 when staged, so a candidate is
+// compared and scored exactly as the rounded model scores the rounded row.
+enum TableKind : int { kTableFull = 0, kTableCompact = 1, kTableHalf = 2 };
+
+struct HalfLayout {
+  uint32_t n_inner;   // nodes in levels [0, D-1)
+  uint32_t off_last;  // byte offset of the last-level 8-byte records
+  uint32_t bytes;     // bytes per tree (multiple of 16)
+};
+
+__host__ __device__ constexpr HalfLayout half_layout(int D) {
+  const uint32_t n_inner = (1u << (D - 1)) - 1u;
+  const uint32_t off_last = (n_inner * 4u + 7u) & ~7u;
+  const uint32_t bytes = (off_last + (1u << (D - 1)) * 8u + 15u) & ~15u;
+  return HalfLayout{n_inner, off_last, bytes};
+}
+
+constexpr uint32_t kHalfFeatureShift = 16;
+constexpr uint32_t kHalfFeatureMask = 0x3FFu;
 
 struct FullLayout {
   uint32_t top;        // levels held as 8-byte records
@@ -192,6 +218,9 @@ struct ScreenShape {
   int group;           // trees walked together per thread (ILP)
   int lanes = 1;       // lanes sharing one candidate (compact walk; CTA = threads * lanes)
   int p_grid = 0;      // full-table P pass: CTAs one wave holds (resident per SM x SMs)
+  int resident = 0;    // full tables: CTAs meant to share an SM (shared memory is padded so
+                       // that no more fit: the block scheduler would otherwise stack tiles
+                       // on some SMs and leave others idle)
 };
 
 // Launch-shape override (mlt_tune_shape, mlt_tune_deep_walk): 0 fields mean
@@ -217,17 +246,23 @@ FullKernelPtr full_kernel_q2(int depth, int group);
 FullDecKernelPtr full_dec_kernel_q2(int depth, int group);
 FullKernelPtr full_kernel_q4(int depth, int group);
 FullDecKernelPtr full_dec_kernel_q4(int depth, int group);
+// traverse_half.cu: half tables (one tree group, stored features only)
+FullKernelPtr half_kernel(int depth, int group);
 
 // traverse.cu
 // n_eff: candidates the pass is expected to walk (used for load balance).
+// half: a half table (binary16 features staged, one tree group)
 ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, int sms,
-                      int device_smem_optin, const ShapeOverride& ov);
+                      int device_smem_optin, const ShapeOverride& ov, bool half);
 ScreenShape plan_compact(int F, long long n_eff, int sms, int device_smem_optin,
                          const ShapeOverride& ov);
 // V pass over n known candidates: the smallest multiple of 32 candidates
 // per CTA (at least 64) that leaves the busiest SM no more tiles than `s`
 // does, so the tiles spread evenly over the SMs.
-ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms);
+ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms, bool half);
+// Pad a full-table shape's shared memory so that at most s.resident CTAs fit
+// on an SM.
+ScreenShape cap_residency(const ScreenShape& s, int optin);
 cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args,
                             const ScreenShape& shape, long long n_tiles, cudaStream_t st);
 // traverse_dec.cu

@@ -44,15 +44,17 @@ FullKernelPtr full_kernel(int depth, int group, int q) {
 //   * a batch of under 32 (64) candidates per SM splits each tile's trees
 //     over 4 (2) groups of warps.
 ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms, int optin,
-                      const ShapeOverride& ov) {
+                      const ShapeOverride& ov, bool half) {
   if (sms < 1) sms = 1;
   if (n_eff < 1) n_eff = 1;
   // tree groups per CTA: a batch of less than a warp (or two) per SM gets
-  // its trees split over 4 (2) groups of warps
-  const int q = ov.lanes ? ov.lanes : n_eff < 32LL * sms ? 4 : n_eff < 64LL * sms ? 2 : 1;
+  // its trees split over 4 (2) groups of warps; half tables walk with one
+  const int q = half ? 1 : ov.lanes ? ov.lanes : n_eff < 32LL * sms ? 4 : n_eff < 64LL * sms ? 2 : 1;
   if (q != 1 && q != 2 && q != 4) return ScreenShape{};
+  if (half && ov.lanes > 1) return ScreenShape{};
+  const int xb = half ? 2 : 4;  // bytes per staged feature
   auto smem_of = [&](int tc, int chunk, int nb) {
-    return full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb, q, chunk);
+    return full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * tb, q, chunk, xb);
   };
   auto fits = [&](size_t smem) { return smem + kStaticSmem <= static_cast<size_t>(optin); };
   auto resident = [&](size_t smem, int tc) {
@@ -96,14 +98,15 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
         best.nbuf = nb;
         best.group = group;
         best.smem = smem;
-        best.p_grid = sms * resident(smem, tc);
+        best.p_grid = sms * std::max(1, res);  // CTAs per wave: the tiles an SM gets, up to residency
+        best.resident = std::max(1, res);
       }
     }
   }
   return best;  // threads == 0: nothing fits
 }
 
-ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms) {
+ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms, bool half) {
   if (s.threads == 0 || n <= 0 || sms < 1) return s;
   const long long tiles_sm = ((n + s.threads - 1) / s.threads + sms - 1) / sms;
   const long long per_tile = (n + sms * tiles_sm - 1) / (sms * tiles_sm);
@@ -113,8 +116,21 @@ ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes,
   ScreenShape b = s;
   b.threads = tc;
   b.smem = full_smem_bytes(F, tc, s.nbuf, static_cast<uint32_t>(s.chunk_trees) * tree_bytes, s.lanes,
-                           s.chunk_trees);
+                           s.chunk_trees, half ? 2 : 4);
   return b;
+}
+
+ScreenShape cap_residency(const ScreenShape& s, int optin) {
+  if (s.threads == 0 || s.resident < 1) return s;
+  const size_t per_cta = kStaticSmem + kCtaReserve;
+  const size_t fit = kSmPerSm / (s.smem + per_cta);
+  if (fit <= static_cast<size_t>(s.resident)) return s;
+  // resident + 1 CTAs of this size cannot fit, whatever the per-CTA
+  // overheads are
+  const size_t need = kSmPerSm / (s.resident + 1) + 1;
+  ScreenShape c = s;
+  if (need + kStaticSmem <= static_cast<size_t>(optin)) c.smem = std::max(s.smem, (need + 15) & ~static_cast<size_t>(15));
+  return c;
 }
 
 // Deep-tree walk: candidates per CTA (TC), lanes per candidate (Q) and trees
@@ -200,13 +216,14 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
   // them on the device (CTAs without rows exit at once)
   TraverseArgs a = args;
   long long ctas = n_tiles;
-  if (args.p_pass && m.kind == kTableFull && shape.p_grid > 0) {
+  if (args.p_pass && m.kind != kTableCompact && shape.p_grid > 0) {
     a.p_wave = shape.p_grid;
     ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
   }
   const dim3 grid(static_cast<unsigned>(ctas));
-  if (m.kind == kTableFull) {
-    FullKernelPtr k = full_kernel(m.depth, shape.group, shape.lanes);
+  if (m.kind != kTableCompact) {
+    FullKernelPtr k = m.kind == kTableHalf ? (shape.lanes == 1 ? half_kernel(m.depth, shape.group) : nullptr)
+                                           : full_kernel(m.depth, shape.group, shape.lanes);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));

@@ -85,6 +85,7 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
   // them on the device (CTAs without rows exit at once)
   TraverseArgs a = args;
   long long ctas = n_tiles;
+  if (m.kind == kTableHalf) return cudaErrorInvalidValue;  // half tables need stored features
   if (args.p_pass && m.kind == kTableFull && shape.p_grid > 0) {
     a.p_wave = shape.p_grid;
     ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;

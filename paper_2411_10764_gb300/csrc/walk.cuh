@@ -22,6 +22,8 @@
 
 #include <cmath>
 
+#include <cuda_fp16.h>
+
 #include "mlt_internal.cuh"
 
 namespace mlt {
@@ -455,23 +457,135 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
 }
 
 // Shared-memory layout of the full-table kernel (host and device agree):
-//   features [F][TC]; rows [TC] u32; nbuf chunk buffers; with Q > 1 tree
-//   groups, two parked-leaf buffers [chunk_trees][TC] fp32; mbarriers.
-__host__ __device__ inline size_t full_smem_rows_off(int F, int TC) {
-  return align_up(static_cast<size_t>(F) * TC * 4, 128);
+//   features [F][TC] (xb = 4 bytes each, 2 for half tables); rows [TC] u32;
+//   nbuf chunk buffers; with Q > 1 tree groups, two parked-leaf buffers
+//   [chunk_trees][TC] fp32; mbarriers.
+__host__ __device__ inline size_t full_smem_rows_off(int F, int TC, int xb = 4) {
+  return align_up(static_cast<size_t>(F) * TC * xb, 128);
 }
-__host__ __device__ inline size_t full_smem_tbuf_off(int F, int TC) {
-  return full_smem_rows_off(F, TC) + align_up(static_cast<size_t>(TC) * 4, 128);
+__host__ __device__ inline size_t full_smem_tbuf_off(int F, int TC, int xb = 4) {
+  return full_smem_rows_off(F, TC, xb) + align_up(static_cast<size_t>(TC) * 4, 128);
 }
-__host__ __device__ inline size_t full_smem_leaf_off(int F, int TC, int nbuf, uint32_t chunk_bytes) {
-  return align_up(full_smem_tbuf_off(F, TC) + static_cast<size_t>(nbuf) * chunk_bytes, 16);
+__host__ __device__ inline size_t full_smem_leaf_off(int F, int TC, int nbuf, uint32_t chunk_bytes, int xb = 4) {
+  return align_up(full_smem_tbuf_off(F, TC, xb) + static_cast<size_t>(nbuf) * chunk_bytes, 16);
 }
 __host__ __device__ inline size_t full_smem_leaf_bytes(int TC, int Q, int chunk_trees) {
   return Q > 1 ? 2 * static_cast<size_t>(chunk_trees) * TC * 4 : 0;
 }
 __host__ __device__ inline size_t full_smem_bytes(int F, int TC, int nbuf, uint32_t chunk_bytes, int Q,
-                                                  int chunk_trees) {
-  return full_smem_leaf_off(F, TC, nbuf, chunk_bytes) + full_smem_leaf_bytes(TC, Q, chunk_trees) + 8 * 4;
+                                                  int chunk_trees, int xb = 4) {
+  return full_smem_leaf_off(F, TC, nbuf, chunk_bytes, xb) + full_smem_leaf_bytes(TC, Q, chunk_trees) + 8 * 4;
+}
+
+// ---------------------------------------------------------------------------
+// Half-table walk (binary16 thresholds, leaves and staged features)
+// ---------------------------------------------------------------------------
+// Stage this thread's candidate as binary16 (round to nearest even; NaN
+// stays NaN, magnitudes past 65504 become infinities).  Returns whether the
+// row holds a NaN.
+__device__ __forceinline__ bool stage_row_half(const TraverseArgs& a, unsigned short* xs, const uint32_t* rowidx,
+                                               long long tile0, int rows_here, int TC) {
+  const int F = a.F;
+  const int c = threadIdx.x;
+  if (c >= rows_here) {
+    for (int f = 0; f < F; ++f) xs[f * TC + c] = 0;
+    return false;
+  }
+  const long long pos = a.p_pass ? static_cast<long long>(rowidx[c]) : tile0 + c;
+  const float* src = a.feats + pos * F;
+  bool nan = false;
+  if (a.vec4) {
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    for (int q = 0; q < (F >> 2); ++q) {
+      const float4 v = ldg_f4_hint(s4 + q, policy_evict_first());
+      const int f = q << 2;
+      xs[(f + 0) * TC + c] = __half_as_ushort(__float2half_rn(v.x));
+      xs[(f + 1) * TC + c] = __half_as_ushort(__float2half_rn(v.y));
+      xs[(f + 2) * TC + c] = __half_as_ushort(__float2half_rn(v.z));
+      xs[(f + 3) * TC + c] = __half_as_ushort(__float2half_rn(v.w));
+      nan |= (v.x != v.x) | (v.y != v.y) | (v.z != v.z) | (v.w != v.w);
+    }
+  } else {
+    for (int f = 0; f < F; ++f) {
+      const float x = __ldg(src + f);
+      xs[f * TC + c] = __half_as_ushort(__float2half_rn(x));
+      nan |= (x != x);
+    }
+  }
+  return nan;
+}
+
+__device__ __forceinline__ unsigned short lds_u16(uint32_t a) {
+  unsigned short v;
+  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
+  return v;
+}
+
+// Go right?  x >= threshold in binary16; a missing x takes the node's
+// default side (bit 31 of the node word).
+template <bool NANP>
+__device__ __forceinline__ uint32_t go_right_half(unsigned short x, uint32_t w) {
+  const __half xh = __ushort_as_half(x);
+  uint32_t right = __hge(xh, __ushort_as_half(static_cast<unsigned short>(w & 0xFFFFu))) ? 1u : 0u;
+  if (NANP && __hisnan(xh) && !(w >> 31)) right = 1u;
+  return right;
+}
+
+// Walk trees [0, nt) of a half-table chunk at shared address tb; xa = shared
+// address of this thread's binary16 feature column (feature f at xa + f *
+// row_bytes).  Leaves (binary16, exact in fp32) are added in tree order.
+template <int D, int G, bool NANP>
+__device__ __forceinline__ float walk_chunk_half(uint32_t tb, int nt, uint32_t tree_bytes, uint32_t xa,
+                                                 uint32_t row_bytes, float acc) {
+  constexpr HalfLayout L = half_layout(D);
+  constexpr uint32_t kLast = L.off_last - L.n_inner * 8u;
+  int t = 0;
+  for (; t + G <= nt; t += G) {
+    uint32_t base[G], j[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      base[g] = tb + static_cast<uint32_t>(t + g) * tree_bytes;
+      j[g] = 0;
+    }
+#pragma unroll
+    for (int l = 0; l < D - 1; ++l) {
+      uint32_t w[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) w[g] = lds_u32(base[g] + j[g] * 4u);
+      unsigned short x[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+        x[g] = lds_u16(((w[g] >> kHalfFeatureShift) & kHalfFeatureMask) * row_bytes + xa);
+#pragma unroll
+      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right_half<NANP>(x[g], w[g]);
+    }
+    uint2 r[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) r[g] = lds_u2(base[g] + kLast + j[g] * 8u);
+    unsigned short x[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) x[g] = lds_u16(((r[g].x >> kHalfFeatureShift) & kHalfFeatureMask) * row_bytes + xa);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const uint32_t bits = go_right_half<NANP>(x[g], r[g].x) ? (r[g].y >> 16) : (r[g].y & 0xFFFFu);
+      acc += __half2float(__ushort_as_half(static_cast<unsigned short>(bits)));
+    }
+  }
+  for (; t < nt; ++t) {
+    const uint32_t base = tb + static_cast<uint32_t>(t) * tree_bytes;
+    uint32_t j = 0;
+#pragma unroll
+    for (int l = 0; l < D - 1; ++l) {
+      const uint32_t w = lds_u32(base + j * 4u);
+      const unsigned short x = lds_u16(((w >> kHalfFeatureShift) & kHalfFeatureMask) * row_bytes + xa);
+      j = 2u * j + 1u + go_right_half<NANP>(x, w);
+    }
+    const uint2 r = lds_u2(base + kLast + j * 8u);
+    const unsigned short x = lds_u16(((r.x >> kHalfFeatureShift) & kHalfFeatureMask) * row_bytes + xa);
+    const uint32_t bits = go_right_half<NANP>(x, r.x) ? (r.y >> 16) : (r.y & 0xFFFFu);
+    acc += __half2float(__ushort_as_half(static_cast<unsigned short>(bits)));
+  }
+  return acc;
 }
 
 // Even split of `len` items into `parts` contiguous pieces whose sizes
@@ -516,8 +630,10 @@ __device__ __forceinline__ void cta_tile(const TraverseArgs& a, long long count,
 // order one chunk later (two leaf buffers), so the sum is the same
 // sequential fp32 sum as with one walker.  More groups put more warps on a
 // small batch; all lanes of a warp still walk the same tree.
-template <int D, int G, int Q>
+template <int D, int G, int Q, bool H = false>
 __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
+  static_assert(!H || Q == 1, "half tables walk with one tree group");
+  constexpr int xb = H ? 2 : 4;  // bytes per staged feature
   extern __shared__ __align__(128) unsigned char smem[];
   const int TC = blockDim.x / Q;
   const int tid = threadIdx.x;
@@ -535,10 +651,10 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   if (rows_here <= 0) return;  // whole CTA, before any copy is issued
 
   float* xs = reinterpret_cast<float*>(smem);
-  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + full_smem_rows_off(a.F, TC));
-  unsigned char* tbuf = smem + full_smem_tbuf_off(a.F, TC);
+  uint32_t* rowidx = reinterpret_cast<uint32_t*>(smem + full_smem_rows_off(a.F, TC, xb));
+  unsigned char* tbuf = smem + full_smem_tbuf_off(a.F, TC, xb);
   const uint32_t chunk_bytes = static_cast<uint32_t>(a.chunk_trees) * a.tree_bytes;
-  const size_t leaf_off = full_smem_leaf_off(a.F, TC, a.nbuf, chunk_bytes);
+  const size_t leaf_off = full_smem_leaf_off(a.F, TC, a.nbuf, chunk_bytes, xb);
   unsigned long long* bars = reinterpret_cast<unsigned long long*>(
       smem + leaf_off + full_smem_leaf_bytes(TC, Q, a.chunk_trees));
   const int n_chunks = (a.n_trees + a.chunk_trees - 1) / a.chunk_trees;
@@ -564,15 +680,19 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   if (a.p_pass && tid < rows_here) rowidx[tid] = a.rows[tile0 + tid];
   // group 0 stages one row per thread (a thread reads only its own rowidx
   // entry); every group reads the same feature columns
-  const bool nan = __syncthreads_or(tid < TC && stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
+  bool nan;
+  if constexpr (H)
+    nan = __syncthreads_or(stage_row_half(a, reinterpret_cast<unsigned short*>(xs), rowidx, tile0, rows_here, TC));
+  else
+    nan = __syncthreads_or(tid < TC && stage_row(a, dec, xs, rowidx, tile0, rows_here, TC));
   // warps past the tile's rows walk zero features: a branch around their
   // walk measured slower than the idle work (it changes the code of the
   // walk loop)
   const bool live = (c & ~31) < rows_here;
 
   float acc = 0.0f;
-  const uint32_t row_bytes = static_cast<uint32_t>(TC) * 4u;
-  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(c) * 4u;
+  const uint32_t row_bytes = static_cast<uint32_t>(TC) * xb;
+  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(c) * xb;
   const uint32_t tbuf_a = smem_u32(tbuf);
   // parked leaves: buffer p holds leaf t of candidate c at la[p] + t * row_bytes
   const uint32_t la0 = smem_u32(smem + leaf_off) + static_cast<uint32_t>(c) * 4u;
@@ -594,8 +714,12 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     const uint32_t tb = tbuf_a + static_cast<uint32_t>(b) * chunk_bytes;
     const int nt = min(a.chunk_trees, a.n_trees - ch * a.chunk_trees);
     const uint32_t la = la0 + static_cast<uint32_t>(ch & 1) * la_step;
-    acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
-              : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);
+    if constexpr (H)
+      acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
+                : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+    else
+      acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
+                : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);
     if (Q > 1 && q == 0 && ch > 0) {
       // the previous chunk's leaves (complete since the last barrier)
       const uint32_t lp = la0 + static_cast<uint32_t>((ch - 1) & 1) * la_step;
@@ -623,6 +747,28 @@ template <int D, int G, int Q>
 __global__ void __launch_bounds__(256)
     k_traverse_full_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
   traverse_full_body<D, G, Q>(a, &d);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(256) k_traverse_half(const __grid_constant__ TraverseArgs a) {
+  traverse_full_body<D, G, 1, true>(a, nullptr);
+}
+
+template <int G>
+FullKernelPtr half_kernel_for(int d) {
+  switch (d) {
+    case 1: return k_traverse_half<1, G>;
+    case 2: return k_traverse_half<2, G>;
+    case 3: return k_traverse_half<3, G>;
+    case 4: return k_traverse_half<4, G>;
+    case 5: return k_traverse_half<5, G>;
+    case 6: return k_traverse_half<6, G>;
+    case 7: return k_traverse_half<7, G>;
+    case 8: return k_traverse_half<8, G>;
+    case 9: return k_traverse_half<9, G>;
+    case 10: return k_traverse_half<10, G>;
+    default: return nullptr;
+  }
 }
 
 // Kernel of depth d (1..10) for G trees in flight and Q tree groups.

@@ -57,6 +57,7 @@ def lib(build_if_missing: bool = True):
         sig = {
             "mlt_set_num_features": [i32],
             "mlt_load_ensemble": [i32, P, i32, i32],
+            "mlt_load_ensemble_f16": [i32, P, i32, i32],
             "mlt_free_ensemble": [i32],
             "mlt_validity_cut": [f32, P],
             "mlt_screen": [P, P, i64, f32, i32, P, P, P],
@@ -124,6 +125,17 @@ def load_ensemble(model_id: int, nodes: np.ndarray, n_trees: int, depth: int) ->
     if nodes.size != n_trees * ((2 << depth) - 1):
         raise ValueError("node array size does not match n_trees and depth")
     _check(lib().mlt_load_ensemble(int(model_id), nodes.ctypes.data, int(n_trees), int(depth)))
+
+
+def load_ensemble_f16(model_id: int, nodes: np.ndarray, n_trees: int, depth: int) -> None:
+    """Load model V or P as half tables (binary16 thresholds, leaves and
+    staged features: changes results, see mlt_load_ensemble_f16)."""
+    nodes = np.ascontiguousarray(nodes)
+    if nodes.dtype.itemsize != 12:
+        raise ValueError("nodes must use the 12-byte slot layout")
+    if nodes.size != n_trees * ((2 << depth) - 1):
+        raise ValueError("node array size does not match n_trees and depth")
+    _check(lib().mlt_load_ensemble_f16(int(model_id), nodes.ctypes.data, int(n_trees), int(depth)))
 
 
 def free_ensemble(model_id: int) -> None:
@@ -334,8 +346,10 @@ def kernel_launches() -> int:
     return int(lib().mlt_kernel_launches())
 
 
-def load_workload_models(w) -> None:
-    """Set F and load the workload's V and P ensembles."""
+def load_workload_models(w, half: bool = False) -> None:
+    """Set F and load the workload's V and P ensembles (as half tables if
+    `half`)."""
     set_num_features(w.cfg.F if w.feats is None else w.feats.shape[1])
-    load_ensemble(MLT_MODEL_V, w.v.nodes, w.v.n_trees, w.v.depth)
-    load_ensemble(MLT_MODEL_P, w.p.nodes, w.p.n_trees, w.p.depth)
+    load = load_ensemble_f16 if half else load_ensemble
+    load(MLT_MODEL_V, w.v.nodes, w.v.n_trees, w.v.depth)
+    load(MLT_MODEL_P, w.p.nodes, w.p.n_trees, w.p.depth)

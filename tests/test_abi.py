@@ -143,3 +143,23 @@ def test_walk_tuning_accepts_and_releases():
     mlt.tune_walk(mlt.MLT_MODEL_P, 64, 4, 8, 8, 2)
     mlt.tune_walk(mlt.MLT_MODEL_P, 96, 2, 2, 16, 3)
     mlt.tune_walk(mlt.MLT_MODEL_P)
+
+
+@pytest.mark.parametrize("case", ["model_a", "depth_11", "leaf_past_binary16", "invalid_tree"])
+def test_half_table_loader_rejects(case):
+    mlt.set_num_features(4)
+    nodes, n_trees, depth, model = _stump(), 1, 1, mlt.MLT_MODEL_P
+    if case == "model_a":
+        model = mlt.MLT_MODEL_A
+    elif case == "depth_11":
+        depth = 11
+        nodes = np.zeros((2 << 11) - 1, mlt.NODE_DTYPE)
+        nodes[0] = (-1, 0.5, 0, (0, 0, 0))
+        nodes["feature"][1:] = -2
+    elif case == "leaf_past_binary16":
+        nodes = _stump(left=65520.0)
+    elif case == "invalid_tree":
+        nodes[0]["feature"] = 9
+    with pytest.raises(mlt.MltError) as e:
+        mlt.load_ensemble_f16(model, nodes, n_trees, depth)
+    assert e.value.code == -1

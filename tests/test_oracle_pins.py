@@ -335,3 +335,59 @@ def test_sa_step_proposals_change_one_knob():
         else:
             assert nxt[i] == parent[i] and np.isneginf(nsc[i])
     del pk
+
+
+# ---------------------------------------------------------------------------
+# Half tables: the binary16 rounding the variant applies (IEEE 754 binary16:
+# 1 sign, 5 exponent, 10 fraction bits; round to nearest, ties to even).
+# Expected values worked by hand from that definition.
+# ---------------------------------------------------------------------------
+HALF_CASES = [
+    (1.0, 1.0),
+    (0.1, 0.0999755859375),              # 0x2E66: 1638/16384
+    (1.0 + 2.0 ** -11, 1.0),             # tie between 1 and 1 + 2^-10: even fraction wins
+    (1.0 + 3 * 2.0 ** -11, 1.0 + 2.0 ** -9),  # tie between fractions 1 and 2: 2 is even
+    (1.0 + 2.0 ** -11 + 2.0 ** -20, 1.0 + 2.0 ** -10),  # just above the tie
+    (65504.0, 65504.0),                  # largest finite
+    (65519.0, 65504.0),
+    (65520.0, np.inf),                   # the tie with 2^16 rounds to infinity
+    (-70000.0, -np.inf),
+    (2.0 ** -24, 2.0 ** -24),            # smallest subnormal
+    (2.0 ** -25, 0.0),                   # tie with 0: even (0) wins
+    (3 * 2.0 ** -26, 2.0 ** -24),
+    (-0.0, -0.0),
+    (1025.0, 1025.0),                    # spacing is 1 in [1024, 2048)
+    (2049.0, 2048.0),                    # spacing 2 in [2048, 4096): tie, 2048 is even
+    (2051.0, 2052.0),                    # tie between 2050 and 2052: 2052 is even
+]
+
+
+@pytest.mark.parametrize("x,expect", HALF_CASES)
+def test_round_half_hand_worked(x, expect):
+    got = O.round_half(np.float32(x))
+    assert got.dtype == np.float32
+    assert float(got) == expect and np.signbit(got) == np.signbit(np.float64(expect))
+
+
+def test_round_half_keeps_nan_and_infinities():
+    got = O.round_half(np.array([np.nan, np.inf, -np.inf], np.float32))
+    assert np.isnan(got[0]) and got[1] == np.inf and got[2] == -np.inf
+
+
+def test_round_half_is_monotone_and_idempotent():
+    rng = np.random.default_rng(7)
+    x = np.sort(rng.standard_normal(100000).astype(np.float32) * rng.choice([1e-3, 1.0, 1e3], 100000))
+    h = O.round_half(x)
+    assert np.all(np.diff(h.astype(np.float64)) >= 0)
+    assert np.array_equal(O.round_half(h), h)
+
+
+def test_half_ensemble_rounds_values_only():
+    w = W.make_workload(2, seed=1, n=1000)
+    nodes, n_trees, depth = O.half_ensemble(w.v)
+    assert (n_trees, depth) == (w.v.n_trees, w.v.depth)
+    assert np.array_equal(nodes["feature"], w.v.nodes["feature"])
+    assert np.array_equal(nodes["default_left"], w.v.nodes["default_left"])
+    used = nodes["feature"] != W.UNUSED
+    assert np.array_equal(nodes["value"][used], O.round_half(w.v.nodes["value"][used]))
+    assert np.array_equal(nodes["value"][~used], w.v.nodes["value"][~used])
