@@ -413,10 +413,29 @@ def run_ours(args):
     for _ in range(3):
         e2e_step()
     e2e_steps = max(10, min(args.steps, 200 if n <= (1 << 20) else 10))
+    # one synchronous call per batch (upload, screen, download in turn)
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
         e2e_step()
-    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    e2e_sync_s = (time.perf_counter() - t0) / e2e_steps
+    e2e_s = e2e_sync_s
+    e2e_how = "mlt_screen_host: one synchronous call per batch"
+    if d is None:
+        # the pipelined entry point: every batch still uploads its features
+        # and downloads its results, overlapped with the previous / next
+        # batch's screening (two pinned result sets in turn)
+        outs2 = [out, (torch.empty(n, dtype=torch.float32).pin_memory().numpy(),
+                       torch.empty(n, dtype=torch.float32).pin_memory().numpy(),
+                       torch.empty(k, dtype=torch.int64).pin_memory().numpy())]
+        outs_b = [outs2[i & 1] for i in range(e2e_steps)]
+        mlt.screen_host_batches([hxn] * 4, thr, k, outs=outs_b[:4], stream=stream)
+        t0 = time.perf_counter()
+        mlt.screen_host_batches([hxn] * e2e_steps, thr, k, outs=outs_b, stream=stream)
+        pipe_s = (time.perf_counter() - t0) / e2e_steps
+        if pipe_s < e2e_s:
+            e2e_s = pipe_s
+            e2e_how = (f"mlt_screen_host_batches: {e2e_steps} host batches in one call, each uploaded and "
+                       f"downloaded, copies overlapped with screening")
     if dist is not None:
         t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -509,7 +528,8 @@ def run_ours(args):
         },
         "e2e": {"value": world * n / e2e_s, "unit": "candidates/s",
                 "h2d_bytes_per_step": h2d_bytes,
-                "d2h_bytes_per_step": int(2 * n * 4 + k * 8)},
+                "d2h_bytes_per_step": int(2 * n * 4 + k * 8),
+                "how": e2e_how, "sync_call_value": world * n / e2e_sync_s},
         "gpu_launches": int(launches),
         "rerank": rerank,
         "half_tables": half,

@@ -184,6 +184,21 @@ int mlt_screen_noalloc(void *stream, const float *feats, int64_t n, float thr, i
 int mlt_screen_host(void *stream, const float *feats_host, int64_t n, float thr, int k,
                     float *pvalid_host, float *perf_host, int64_t *topk_host);
 
+/* mlt_screen over n_batches independent host batches of n candidates each,
+ * pipelined: batch b is screened on `stream` while a library-owned copy
+ * stream returns batch b-1's results and uploads batch b+1 (two device
+ * staging sets in turn).  Each batch's results are exactly mlt_screen's.
+ *   feats_host[b]   host [n][F] fp32 (page-locked memory lets the copies
+ *                   overlap the screening)
+ *   pvalid_host, perf_host: NULL, or arrays of n_batches host pointers to
+ *                   [n] fp32 (a NULL entry skips that batch's copy)
+ *   topk_host[b]    host [k] int64
+ * The pointer arrays are read during the call only.  Synchronous: returns
+ * when every result is on the host. */
+int mlt_screen_host_batches(void *stream, int64_t n_batches, const float *const *feats_host, int64_t n,
+                            float thr, int k, float *const *pvalid_host, float *const *perf_host,
+                            int64_t *const *topk_host);
+
 /* Batched accumulation (Sec. 2: the explorer applies models P and V until
  * it has accumulated (alpha+1)N configurations): candidates 0 .. n_total-1
  * are screened in consecutive batches of `batch`; after each batch the

@@ -100,6 +100,17 @@ struct ScratchOwner {
   float* h_pvalid = nullptr;
   float* h_perf = nullptr;
   int64_t* h_topk = nullptr;
+  // pipelined host batches: two staging sets, a copy stream and its events
+  long long hb_cap_n = -1;
+  int hb_cap_F = 0;
+  float* hb_feats[2] = {nullptr, nullptr};
+  float* hb_pvalid[2] = {nullptr, nullptr};
+  float* hb_perf[2] = {nullptr, nullptr};
+  int64_t* hb_topk[2] = {nullptr, nullptr};
+  cudaStream_t hb_copy = nullptr;
+  cudaEvent_t hb_in[2] = {nullptr, nullptr};    // batch's features are on the device
+  cudaEvent_t hb_out[2] = {nullptr, nullptr};   // batch's screening is done
+  cudaEvent_t hb_down[2] = {nullptr, nullptr};  // batch's results are on the host
 };
 
 std::mutex g_mu;
@@ -993,6 +1004,108 @@ int mlt_screen_host(void* stream, const float* feats_host, int64_t n, float thr,
   }
   MLT_CUDA(cudaMemcpyAsync(topk_host, S.h_topk, sizeof(int64_t) * k, cudaMemcpyDeviceToHost, st), "top-k download");
   MLT_CUDA(cudaStreamSynchronize(st), "stream synchronize");
+  return MLT_OK;
+}
+
+int mlt_screen_host_batches(void* stream, int64_t n_batches, const float* const* feats_host, int64_t n, float thr,
+                            int k, float* const* pvalid_host, float* const* perf_host, int64_t* const* topk_host) {
+  int rc = check_screen_args(n, thr, k);
+  if (rc != MLT_OK) return rc;
+  if (n_batches < 0) return fail(MLT_EINVAL, "n_batches must be >= 0");
+  if (n_batches == 0) return MLT_OK;
+  if (feats_host == nullptr || topk_host == nullptr) return fail(MLT_EINVAL, "feats_host and topk_host must be non-NULL");
+  for (int64_t b = 0; b < n_batches; ++b)
+    if ((n > 0 && feats_host[b] == nullptr) || topk_host[b] == nullptr)
+      return fail(MLT_EINVAL, "batch %lld: host buffers must be non-NULL", static_cast<long long>(b));
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  cudaStream_t sc = static_cast<cudaStream_t>(stream);
+  ScratchOwner& S = g_scr;
+  if (S.hb_copy == nullptr) {
+    MLT_CUDA(cudaStreamCreateWithFlags(&S.hb_copy, cudaStreamNonBlocking), "copy stream");
+    for (int i = 0; i < 2; ++i) {
+      MLT_CUDA(cudaEventCreateWithFlags(&S.hb_in[i], cudaEventDisableTiming), "cudaEventCreate");
+      MLT_CUDA(cudaEventCreateWithFlags(&S.hb_out[i], cudaEventDisableTiming), "cudaEventCreate");
+      MLT_CUDA(cudaEventCreateWithFlags(&S.hb_down[i], cudaEventDisableTiming), "cudaEventCreate");
+    }
+  }
+  if (n > S.hb_cap_n || g_F != S.hb_cap_F) {
+    cudaDeviceSynchronize();
+    for (int i = 0; i < 2; ++i) {
+      cudaFree(S.hb_feats[i]);
+      cudaFree(S.hb_pvalid[i]);
+      cudaFree(S.hb_perf[i]);
+      cudaFree(S.hb_topk[i]);
+      S.hb_feats[i] = nullptr;
+      S.hb_pvalid[i] = S.hb_perf[i] = nullptr;
+      S.hb_topk[i] = nullptr;
+    }
+    S.hb_cap_n = -1;
+    const long long cap = n < 1024 ? 1024 : n;
+    for (int i = 0; i < 2; ++i) {
+      if (cudaMalloc(&S.hb_feats[i], sizeof(float) * cap * g_F) != cudaSuccess ||
+          cudaMalloc(&S.hb_pvalid[i], sizeof(float) * cap) != cudaSuccess ||
+          cudaMalloc(&S.hb_perf[i], sizeof(float) * cap) != cudaSuccess ||
+          cudaMalloc(&S.hb_topk[i], sizeof(int64_t) * kMaxK) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(MLT_ENOMEM, "cannot allocate device staging for host batches");
+      }
+    }
+    S.hb_cap_n = cap;
+    S.hb_cap_F = g_F;
+  }
+  rc = ensure_scratch(n);  // before the pipeline: growing it synchronises the device
+  if (rc != MLT_OK) return rc;
+  cudaStream_t sh = S.hb_copy;
+  const size_t in_bytes = sizeof(float) * static_cast<size_t>(n) * g_F;
+  auto upload = [&](int64_t b) -> int {
+    const int i = static_cast<int>(b & 1);
+    if (n > 0)
+      MLT_CUDA(cudaMemcpyAsync(S.hb_feats[i], feats_host[b], in_bytes, cudaMemcpyHostToDevice, sh), "feature upload");
+    MLT_CUDA(cudaEventRecord(S.hb_in[i], sh), "cudaEventRecord");
+    return MLT_OK;
+  };
+  auto download = [&](int64_t b) -> int {
+    const int i = static_cast<int>(b & 1);
+    MLT_CUDA(cudaStreamWaitEvent(sh, S.hb_out[i], 0), "cudaStreamWaitEvent");
+    if (n > 0 && pvalid_host != nullptr && pvalid_host[b] != nullptr)
+      MLT_CUDA(cudaMemcpyAsync(pvalid_host[b], S.hb_pvalid[i], sizeof(float) * n, cudaMemcpyDeviceToHost, sh),
+               "pvalid download");
+    if (n > 0 && perf_host != nullptr && perf_host[b] != nullptr)
+      MLT_CUDA(cudaMemcpyAsync(perf_host[b], S.hb_perf[i], sizeof(float) * n, cudaMemcpyDeviceToHost, sh),
+               "perf download");
+    MLT_CUDA(cudaMemcpyAsync(topk_host[b], S.hb_topk[i], sizeof(int64_t) * k, cudaMemcpyDeviceToHost, sh),
+             "top-k download");
+    MLT_CUDA(cudaEventRecord(S.hb_down[i], sh), "cudaEventRecord");
+    return MLT_OK;
+  };
+  // the copy stream starts after the caller's earlier work on `stream`
+  MLT_CUDA(cudaEventRecord(S.hb_out[1], sc), "cudaEventRecord");
+  MLT_CUDA(cudaStreamWaitEvent(sh, S.hb_out[1], 0), "cudaStreamWaitEvent");
+  rc = upload(0);
+  if (rc != MLT_OK) return rc;
+  // batch b screens on `stream` while the copy stream brings back batch
+  // b-1's results and uploads batch b+1 (two staging sets in turn)
+  for (int64_t b = 0; b < n_batches; ++b) {
+    const int i = static_cast<int>(b & 1);
+    MLT_CUDA(cudaStreamWaitEvent(sc, S.hb_in[i], 0), "cudaStreamWaitEvent");
+    if (b >= 2) MLT_CUDA(cudaStreamWaitEvent(sc, S.hb_down[i], 0), "cudaStreamWaitEvent");
+    rc = run_screen_with(sc, S.hb_feats[i], nullptr, n, thr, k, S.hb_pvalid[i], S.hb_perf[i], S.hb_topk[i], S.s, true);
+    if (rc != MLT_OK) return rc;
+    MLT_CUDA(cudaEventRecord(S.hb_out[i], sc), "cudaEventRecord");
+    if (b >= 1) {
+      rc = download(b - 1);  // waits for batch b-1, whose staging batch b+1 reuses
+      if (rc != MLT_OK) return rc;
+    }
+    if (b + 1 < n_batches) {
+      rc = upload(b + 1);
+      if (rc != MLT_OK) return rc;
+    }
+  }
+  rc = download(n_batches - 1);
+  if (rc != MLT_OK) return rc;
+  MLT_CUDA(cudaStreamSynchronize(sh), "copy stream synchronize");
+  MLT_CUDA(cudaStreamSynchronize(sc), "stream synchronize");
   return MLT_OK;
 }
 

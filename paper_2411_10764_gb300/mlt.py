@@ -58,6 +58,7 @@ def lib(build_if_missing: bool = True):
             "mlt_set_num_features": [i32],
             "mlt_load_ensemble": [i32, P, i32, i32],
             "mlt_load_ensemble_f16": [i32, P, i32, i32],
+            "mlt_screen_host_batches": [P, i64, P, i64, f32, i32, P, P, P],
             "mlt_free_ensemble": [i32],
             "mlt_validity_cut": [f32, P],
             "mlt_screen": [P, P, i64, f32, i32, P, P, P],
@@ -274,6 +275,28 @@ def screen_host(feats: np.ndarray, thr: float, k: int, out=None, stream=None):
     _check(lib().mlt_screen_host(_stream_ptr(stream), feats.ctypes.data, n, C.c_float(thr), int(k),
                                  pv.ctypes.data, pf.ctypes.data, tk.ctypes.data))
     return pv, pf, tk
+
+
+def screen_host_batches(feats, thr: float, k: int, outs=None, stream=None):
+    """Screen a list of host batches (each [n][F] fp32, page-locked for
+    overlap) with the pipelined host entry point.  `outs`: a list of
+    (pvalid, perf, topk) host arrays per batch (pvalid / perf may be None);
+    allocated if omitted.  Returns the list."""
+    feats = [np.asarray(f) for f in feats]
+    nb = len(feats)
+    n = feats[0].shape[0] if nb else 0
+    for f in feats:
+        if f.dtype != np.float32 or not f.flags.c_contiguous or f.shape[0] != n:
+            raise ValueError("batches must be C-contiguous fp32 arrays of equal length")
+    if outs is None:
+        outs = [(np.empty(n, np.float32), np.empty(n, np.float32), np.empty(k, np.int64)) for _ in range(nb)]
+    arr = lambda xs: (C.c_void_p * max(1, nb))(*[None if x is None else x.ctypes.data for x in xs])
+    fp = arr(feats)
+    pv = arr([o[0] for o in outs])
+    pf = arr([o[1] for o in outs])
+    tk = arr([o[2] for o in outs])
+    _check(lib().mlt_screen_host_batches(_stream_ptr(stream), nb, fp, int(n), C.c_float(thr), int(k), pv, pf, tk))
+    return outs
 
 
 def _decoder_args(radices, option_values, program):

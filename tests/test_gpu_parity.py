@@ -390,3 +390,29 @@ def test_sa_step_reports_parent_past_the_space():
                 1.0, w.thr)
     assert e.value.code == -1
     mlt.sync_status()
+
+
+def test_host_batches_pipeline_matches_oracle():
+    """Pipelined host batches (mlt_screen_host_batches): every batch equals
+    the oracle's screening of it, whatever the overlap; optional outputs
+    may be skipped."""
+    import torch
+
+    w = W.make_workload(2, seed=9, n=20001)
+    mlt.load_workload_models(w)
+    rng = np.random.default_rng(5)
+    batches = [np.ascontiguousarray(w.feats[rng.permutation(w.n)]) for _ in range(5)]
+    pinned = [torch.from_numpy(b).pin_memory().numpy() for b in batches]
+    outs = mlt.screen_host_batches(pinned, w.thr, w.k)
+    for b, (pv, pf, tk) in zip(batches, outs):
+        opv, opf, valid, _ = O.screen_rows(b, w.v, w.p, w.thr, threads=THREADS)
+        otk, s = O.topk(opf, valid, w.k)
+        assert_parity((pv, pf, tk, s), (opv, opf, otk, s))
+    # top-k only, a single batch, then an odd batch count
+    for nb in (1, 3):
+        outs = [(None, None, np.empty(w.k, np.int64)) for _ in range(nb)]
+        outs = mlt.screen_host_batches(pinned[:nb], w.thr, w.k, outs=outs)
+        for b, (_, _, tk) in zip(batches, outs):
+            _, opf, valid, _ = O.screen_rows(b, w.v, w.p, w.thr, threads=THREADS)
+            otk, _ = O.topk(opf, valid, w.k)
+            assert np.array_equal(tk, otk)
