@@ -394,12 +394,14 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
           std::memcpy(dst + lay.off_thr + 4 * (j - lay.n_top), &thr_of[j], 4);
           std::memcpy(dst + lay.off_meta + 4 * (j - lay.n_top), &meta_of[j], 4);
         } else {
-          unsigned char* rec = dst + lay.off_last + 16 * (j - lay.n_inner);
+          const uint32_t q = j - lay.n_inner;
+          unsigned char* rec = dst + lay.off_last + 8 * q;
+          unsigned char* lv = dst + lay.off_last + 8 * (1u << (depth - 1)) + 8 * q;  // leaf pair
           const float left = inherit[2 * j + 1], right = inherit[2 * j + 2];
           std::memcpy(rec, &thr_of[j], 4);
           std::memcpy(rec + 4, &meta_of[j], 4);
-          std::memcpy(rec + 8, &left, 4);
-          std::memcpy(rec + 12, &right, 4);
+          std::memcpy(lv, &left, 4);
+          std::memcpy(lv + 4, &right, 4);
         }
       }
     }

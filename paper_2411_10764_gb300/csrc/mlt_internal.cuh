@@ -37,9 +37,11 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 //                          nodes, mostly broadcast reads;
 //   levels [top, D-1)    : thresholds and metas in two 4-byte arrays -- a
 //                          32-lane gather of 4-byte words;
-//   level D-1 (last)     : 16-byte records {threshold, meta, left leaf,
-//                          right leaf} -- the last split and both leaves in
-//                          one load.
+//   level D-1 (last)     : 8-byte records {threshold, meta}, then the 2^D
+//                          leaves (leaf pair of last-level node q at 2q):
+//                          only the chosen leaf is read, which costs fewer
+//                          shared-memory wavefronts than one 16-byte record
+//                          holding both.
 // A shallower leaf is replicated into every leaf slot below it (its
 // pass-through nodes test feature 0; any path gives the leaf).
 //
@@ -84,7 +86,7 @@ struct FullLayout {
   uint32_t n_inner;    // nodes in levels [0, D-1)
   uint32_t off_thr;    // byte offset of the middle-level thresholds
   uint32_t off_meta;   // byte offset of the middle-level metas
-  uint32_t off_last;   // byte offset of the last-level 16-byte records
+  uint32_t off_last;   // byte offset of the last-level 8-byte records (the leaves follow them)
   uint32_t bytes;      // bytes per tree (multiple of 16)
 };
 
@@ -95,6 +97,7 @@ __host__ __device__ constexpr FullLayout full_layout(int D) {
   const uint32_t off_thr = n_top * 8u;
   const uint32_t off_meta = off_thr + (n_inner - n_top) * 4u;
   const uint32_t off_last = (off_meta + (n_inner - n_top) * 4u + 15u) & ~15u;
+  // last level: 2^(D-1) 8-byte {threshold, meta} records, then 2^D leaves
   const uint32_t bytes = off_last + (1u << (D - 1)) * 16u;
   return FullLayout{top, n_top, n_inner, off_thr, off_meta, off_last, bytes};
 }

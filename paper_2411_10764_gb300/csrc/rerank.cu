@@ -41,9 +41,10 @@ __device__ float leaf_full(const unsigned char* tree, int D, const float* x) {
     const float xv = __ldg(x + (meta & ~kMetaDefaultLeft));
     j = 2u * j + 1u + go_right_nan(xv, thr, meta);
   }
-  const uint4 r = __ldg(reinterpret_cast<const uint4*>(tree + L.off_last) + (j - L.n_inner));
+  const uint2 r = __ldg(reinterpret_cast<const uint2*>(tree + L.off_last) + (j - L.n_inner));
   const float xv = __ldg(x + (r.y & ~kMetaDefaultLeft));
-  return __uint_as_float(go_right_nan(xv, r.x, r.y) ? r.w : r.z);
+  const float* lv = reinterpret_cast<const float*>(tree + L.off_last + 8u * (1u << (D - 1)));
+  return __ldg(lv + 2u * (j - L.n_inner) + go_right_nan(xv, r.x, r.y));
 }
 
 // One tree of a compact table (breadth-first records).

@@ -382,7 +382,8 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
   // byte offsets folded with the heap index of each region's first node
   constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
   constexpr uint32_t kMeta = L.off_meta - L.n_top * 4u;
-  constexpr uint32_t kLast = L.off_last - L.n_inner * 16u;
+  constexpr uint32_t kLast = L.off_last - L.n_inner * 8u;
+  constexpr uint32_t kLeaf = L.off_last + (1u << (D - 1)) * 8u - L.n_inner * 8u;
   int t = q;
   for (; t + (G - 1) * Q < nt; t += G * Q) {
     uint32_t base[G], j[G];
@@ -413,15 +414,18 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
 #pragma unroll
       for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], thr[g], meta[g]);
     }
-    uint4 r[G];
+    uint2 r[G];
 #pragma unroll
-    for (int g = 0; g < G; ++g) r[g] = lds_u4(base[g] + kLast + j[g] * 16u);
+    for (int g = 0; g < G; ++g) r[g] = lds_u2(base[g] + kLast + j[g] * 8u);
     float x[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
+    float lf[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) lf[g] = lds_f32(base[g] + kLeaf + (2u * j[g] + go_right<NANP>(x[g], r[g].x, r[g].y)) * 4u);
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      const float leaf = __uint_as_float(go_right<NANP>(x[g], r[g].x, r[g].y) ? r[g].w : r[g].z);
+      const float leaf = lf[g];
       if (Q == 1)
         acc += leaf;
       else
@@ -445,9 +449,9 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
       const float x = lds_f32(meta * row_bytes + xa);
       j = 2u * j + 1u + go_right<NANP>(x, thr, meta);
     }
-    const uint4 r = lds_u4(base + kLast + j * 16u);
+    const uint2 r = lds_u2(base + kLast + j * 8u);
     const float x = lds_f32(r.y * row_bytes + xa);
-    const float leaf = __uint_as_float(go_right<NANP>(x, r.x, r.y) ? r.w : r.z);
+    const float leaf = lds_f32(base + kLeaf + (2u * j + go_right<NANP>(x, r.x, r.y)) * 4u);
     if (Q == 1)
       acc += leaf;
     else
