@@ -5,17 +5,20 @@
 // regressor over the visible and the compiler's hidden features, deeper
 // than P (depth 14, Table 3) -- picks the final N from them.  The batch is
 // tiny (tens to a few thousand candidates) and the trees deep, so the walk
-// is latency-bound: one warp per candidate, lanes walking different trees
-// straight from global memory (L1/L2), leaves parked in shared memory and
-// added by one lane in tree order (the same exact fp32 sequential sum as
-// the screening walk).  One CTA then sorts the 64-bit keys (score, index).
+// is a chain of dependent loads: one CTA per candidate, its threads walking
+// different trees straight from global memory (L1/L2) -- one tree each when
+// the batch is small enough to spread over the GPU -- leaves parked in
+// shared memory and added by one thread in tree order (the same exact fp32
+// sequential sum as the screening walk).  One CTA then sorts the 64-bit keys
+// (score, index).
+#include <algorithm>
+
 #include "mlt_internal.cuh"
 
 namespace mlt {
 namespace {
 
-constexpr int kWarpsPerCta = 8;
-constexpr int kTreeChunk = 512;  // leaves parked per warp before summing
+constexpr int kTreeChunk = 1024;  // leaves parked before summing
 constexpr int kSelectThreads = 1024;
 
 __device__ __forceinline__ uint32_t go_right_nan(float x, uint32_t thr_bits, uint32_t meta) {
@@ -75,20 +78,18 @@ struct RerankArgs {
   unsigned* err;
 };
 
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_rerank_walk(const __grid_constant__ RerankArgs a) {
-  __shared__ float parked[kWarpsPerCta][kTreeChunk];
+__global__ void __launch_bounds__(1024) k_rerank_walk(const __grid_constant__ RerankArgs a) {
+  __shared__ float parked[kTreeChunk];
   pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= a.m) return;  // whole warp
+  const int i = blockIdx.x;  // one candidate per CTA
   const long long c = a.cand[i];
   if (c < 0 || c >= a.n) {
-    if (lane == 0) {
+    if (threadIdx.x == 0) {
       a.out_score[i] = -INFINITY;
       a.keys[i] = 0ull;  // sorts below every real key
       if (c >= a.n) atomicOr(a.err, kErrBadIndex);
     }
-    return;
+    return;  // whole CTA
   }
   const float* x = a.feats + c * a.F;
   const uint32_t* offs = reinterpret_cast<const uint32_t*>(a.table);
@@ -96,18 +97,17 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_rerank_walk(const __grid_
   float acc = 0.0f;
   for (int base = 0; base < a.n_trees; base += kTreeChunk) {
     const int nt = min(kTreeChunk, a.n_trees - base);
-    for (int t = lane; t < nt; t += 32) {
+    for (int t = threadIdx.x; t < nt; t += blockDim.x) {
       const int tree = base + t;
-      parked[warp][t] = a.kind == kTableFull
-                            ? leaf_full(a.table + static_cast<size_t>(tree) * a.tree_bytes, a.depth, x)
-                            : leaf_compact(recs + __ldg(offs + tree), x);
+      parked[t] = a.kind == kTableFull ? leaf_full(a.table + static_cast<size_t>(tree) * a.tree_bytes, a.depth, x)
+                                       : leaf_compact(recs + __ldg(offs + tree), x);
     }
-    __syncwarp();
-    if (lane == 0)
-      for (int t = 0; t < nt; ++t) acc += parked[warp][t];  // tree order
-    __syncwarp();
+    __syncthreads();
+    if (threadIdx.x == 0)
+      for (int t = 0; t < nt; ++t) acc += parked[t];  // tree order
+    __syncthreads();
   }
-  if (lane == 0) {
+  if (threadIdx.x == 0) {
     a.out_score[i] = acc;
     const uint32_t u = __float_as_uint(acc == 0.0f ? 0.0f : acc);
     const uint32_t mono = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
@@ -163,8 +163,14 @@ cudaError_t launch_rerank(const DeviceModel& A, const float* feats, int F, long 
     a.out_score = out_score;
     a.keys = keys;
     a.err = err;
-    const unsigned grid = static_cast<unsigned>((m + kWarpsPerCta - 1) / kWarpsPerCta);
-    cudaError_t e = launch_pdl(k_rerank_walk, dim3(grid), dim3(kWarpsPerCta * 32), 0, st, a);
+    // threads per candidate: one per tree (a multiple of 32, at most 1,024),
+    // fewer when the batch would hold more than 2,048 threads per SM
+    int sms = 0, dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const long long fill = std::max(32LL, static_cast<long long>(sms > 0 ? sms : 1) * 2048 / m / 32 * 32);
+    const int threads = static_cast<int>(std::min<long long>({(A.n_trees + 31) / 32 * 32, 1024LL, fill}));
+    cudaError_t e = launch_pdl(k_rerank_walk, dim3(static_cast<unsigned>(m)), dim3(threads), 0, st, a);
     if (e != cudaSuccess) return e;
   }
   int m2 = 1;
