@@ -482,6 +482,64 @@ def run_ours(args):
                         "overlap are against the fp32 run on the same batch"}
         mlt.load_workload_models(w)
 
+    # the next rows of the path: batched accumulation (mlt_screen_until) on
+    # this batch, and the explorer's proposal step (mlt_sa_step) over the
+    # decoded conv2d knob space
+    accumulation = sa = None
+    if not args.no_next and d is None:
+        target = max(k, survivors // 4)
+        batch = max(32, n // 8)
+        for _ in range(3):
+            mlt.screen_until(x, batch, target, thr, k, stream=stream)
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        reps = 20
+        a0.record(stream)
+        for _ in range(reps):
+            _, _, _, st_ = mlt.screen_until(x, batch, target, thr, k, stream=stream)
+        a1.record(stream)
+        torch.cuda.synchronize(dev)
+        mlt.sync_status(stream)
+        consumed, kept, batches = (int(v) for v in st_.cpu().tolist())
+        acc_ms = a0.elapsed_time(a1) / reps
+        accumulation = {"what": f"mlt_screen_until: batches of {batch}, stop once {target} valid candidates are kept",
+                        "ms_per_call": acc_ms, "consumed": consumed, "kept": kept, "batches": batches,
+                        "candidates_per_s": consumed / (acc_ms / 1e3)}
+    if not args.no_next:
+        w4 = W.make_workload(4, seed=seed, n=1)
+        mlt.load_workload_models(w4)
+        dec4 = w4.decoder
+        m_chains = 1 << 20
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(seed)
+        parent = torch.randint(0, dec4.space, (m_chains,), device=dev, dtype=torch.int64, generator=gen)
+        pscore = torch.full((m_chains,), float("-inf"), device=dev)
+        s_steps = 10
+        draws = [(torch.randint(0, 1 << 30, (m_chains,), device=dev, dtype=torch.int32, generator=gen),
+                  torch.randint(0, 1 << 30, (m_chains,), device=dev, dtype=torch.int32, generator=gen),
+                  torch.log(torch.rand(m_chains, device=dev, generator=gen)))
+                 for _ in range(s_steps + 2)]
+        for i in range(2):
+            parent, pscore, _ = mlt.sa_step(dec4.radices, dec4.option_values, dec4.program, parent, pscore,
+                                            *draws[i], 1.0, w4.thr, stream=stream)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        accepted = 0
+        for i in range(2, s_steps + 2):
+            parent, pscore, acc_ = mlt.sa_step(dec4.radices, dec4.option_values, dec4.program, parent, pscore,
+                                               *draws[i], 1.0, w4.thr, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mlt.sync_status(stream)
+        accepted = int(acc_.sum().item())
+        sa_ms = e0.elapsed_time(e1) / s_steps
+        sa = {"what": f"mlt_sa_step: {m_chains} simulated-annealing chains over the conv2d knob space "
+                      f"(decode, V {w4.v.n_trees}x d{w4.v.depth}, P {w4.p.n_trees}x d{w4.p.depth}, Metropolis at T=1)",
+              "ms_per_step": sa_ms, "proposals_per_s": m_chains / (sa_ms / 1e3),
+              "accepted_last_step": accepted / m_chains}
+        mlt.load_workload_models(w)
+
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
@@ -533,6 +591,8 @@ def run_ours(args):
         "gpu_launches": int(launches),
         "rerank": rerank,
         "half_tables": half,
+        "accumulation": accumulation,
+        "sa_step": sa,
         "clocks": clocks,
         "wall_ms_per_step_incl_flush": wall * 1e3 / args.steps,
     }
@@ -559,6 +619,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-rerank", action="store_true")
     ap.add_argument("--no-half", action="store_true", help="skip the half-table variant's timing")
+    ap.add_argument("--no-next", action="store_true",
+                    help="skip the accumulation and explorer-step timings")
     ap.add_argument("--n", type=int, default=None,
                     help="candidates per batch (default: the workload's size; smaller for profiling captures)")
     args = ap.parse_args()
