@@ -219,20 +219,20 @@ struct ScreenShape {
   int chunk_trees;
   int nbuf;
   int group;           // trees walked together per thread (ILP)
-  int lanes = 1;       // lanes sharing one candidate (compact walk; CTA = threads * lanes)
+  int lanes = 1;       // threads sharing one candidate's trees: warp groups (full tables) or
+                       // lanes of a warp (compact tables); CTA = threads * lanes
   int p_grid = 0;      // full-table P pass: CTAs one wave holds (resident per SM x SMs)
   int resident = 0;    // full tables: CTAs meant to share an SM (shared memory is padded so
                        // that no more fit: the block scheduler would otherwise stack tiles
                        // on some SMs and leave others idle)
 };
 
-// Launch-shape override (mlt_tune_shape, mlt_tune_deep_walk): 0 fields mean
-// "choose".
+// Launch-shape override (mlt_tune_walk): 0 fields mean "choose".
 struct ShapeOverride {
-  int threads = 0;
+  int threads = 0;      // candidates per CTA
   int chunk_trees = 0;
   int nbuf = 0;
-  int lanes = 0;
+  int lanes = 0;        // splits
   int group = 0;
 };
 
