@@ -205,7 +205,7 @@ __device__ __forceinline__ bool stage_row(const TraverseArgs& a, const DecodePar
   if (a.vec4) {
     const float4* s4 = reinterpret_cast<const float4*>(src);
     const int F4 = F >> 2;
-    constexpr int U = 4;
+    constexpr int U = 8;
     for (int q0 = 0; q0 < F4; q0 += U) {
       float4 v[U];
 #pragma unroll
