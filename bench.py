@@ -485,7 +485,7 @@ def run_ours(args):
     # the next rows of the path: batched accumulation (mlt_screen_until) on
     # this batch, and the explorer's proposal step (mlt_sa_step) over the
     # decoded conv2d knob space
-    accumulation = sa = None
+    accumulation = sa = decode = None
     if not args.no_next and d is None:
         target = max(k, survivors // 4)
         batch = max(32, n // 8)
@@ -538,6 +538,27 @@ def run_ours(args):
                       f"(decode, V {w4.v.n_trees}x d{w4.v.depth}, P {w4.p.n_trees}x d{w4.p.depth}, Metropolis at T=1)",
               "ms_per_step": sa_ms, "proposals_per_s": m_chains / (sa_ms / 1e3),
               "accepted_last_step": accepted / m_chains}
+        # the knob decoder on its own (mlt_decode_knobs): 2^22 candidates of
+        # the same space materialised as option indices and features, an HBM
+        # write stream
+        n_dec = 1 << 22
+        for _ in range(2):
+            mlt.decode_knobs(dec4.radices, dec4.option_values, dec4.program, 0, n_dec, device=dev, stream=stream)
+        torch.cuda.synchronize(dev)
+        reps = 10
+        e0.record(stream)
+        for i in range(reps):
+            kn, fe = mlt.decode_knobs(dec4.radices, dec4.option_values, dec4.program, (i % 4) * n_dec, n_dec,
+                                      device=dev, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mlt.sync_status(stream)
+        dec_ms = e0.elapsed_time(e1) / reps
+        dec_bytes = kn.numel() * kn.element_size() + fe.numel() * fe.element_size()
+        decode = {"what": f"mlt_decode_knobs: {n_dec} conv2d candidates to {dec4.radices.size} option indices "
+                          f"(u8) and {dec4.program.size} fp32 features each",
+                  "ms_per_call": dec_ms, "candidates_per_s": n_dec / (dec_ms / 1e3),
+                  "bytes_written": int(dec_bytes), "write_gbs": dec_bytes / (dec_ms / 1e3) / 1e9}
         mlt.load_workload_models(w)
 
     if rank != 0:
@@ -593,6 +614,7 @@ def run_ours(args):
         "half_tables": half,
         "accumulation": accumulation,
         "sa_step": sa,
+        "decode_knobs": decode,
         "clocks": clocks,
         "wall_ms_per_step_incl_flush": wall * 1e3 / args.steps,
     }

@@ -34,33 +34,41 @@ CompactDecKernel compact_dec_kernel(int group, int lanes) {
   return nullptr;
 }
 
-// One thread per candidate: decode into a shared-memory column, then write
-// the rows out coalesced.
+// One thread per candidate: decode into a shared-memory column (stride
+// TC + 1, so that both the column writes and the row reads below hit 32
+// different banks), then write the rows out coalesced.
 __global__ void __launch_bounds__(256)
     k_decode_rows(const __grid_constant__ DecodeParams d, long long n, uint8_t* out_knobs, float* out_feats) {
   extern __shared__ __align__(128) unsigned char smem[];
   float* xs = reinterpret_cast<float*>(smem);
   const int TC = blockDim.x, tid = threadIdx.x, F = d.F;
+  const int stride = TC + 1;
   const long long tile0 = static_cast<long long>(blockIdx.x) * TC;
   const int rows_here = static_cast<int>(min(static_cast<long long>(TC), n - tile0));
   if (tid < rows_here) {
     const long long idx = d.first_index + tile0 + tid;
-    decode_column(d, idx, xs, TC, tid);
+    decode_column(d, idx, xs, stride, tid);
     if (out_knobs != nullptr) {
-      long long rem = idx;
-      for (int j = 0; j < d.n_knobs; ++j) {
-        const long long q = rem / d.radix[j];
-        out_knobs[(tile0 + tid) * d.n_knobs + j] = static_cast<uint8_t>(rem - q * d.radix[j]);
-        rem = q;
-      }
+      int digit[kMaxKnobs];
+      knob_digits(d, idx, digit);
+      for (int j = 0; j < d.n_knobs; ++j) out_knobs[(tile0 + tid) * d.n_knobs + j] = static_cast<uint8_t>(digit[j]);
     }
   }
   __syncthreads();
   if (out_feats != nullptr) {
+    // element v = r * F + f of the tile's rows, v = tid, tid + TC, ...:
+    // (r, f) advance by (TC / F, TC % F) with a carry, no division per step
+    const int dr = TC / F, df = TC - dr * F;
+    int r = tid / F, f = tid - r * F;
+    float* dst = out_feats + tile0 * F;
     for (int v = tid; v < rows_here * F; v += TC) {
-      const int r = v / F;
-      const int f = v - r * F;
-      out_feats[(tile0 + r) * F + f] = xs[f * TC + r];
+      dst[v] = xs[f * stride + r];
+      r += dr;
+      f += df;
+      if (f >= F) {
+        f -= F;
+        ++r;
+      }
     }
   }
 }
@@ -115,8 +123,8 @@ cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* ou
                                cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   int tc = 256;
-  while (tc > 32 && static_cast<size_t>(dec.F) * tc * 4 > 200 * 1024) tc >>= 1;
-  const size_t smem = static_cast<size_t>(dec.F) * tc * 4;
+  while (tc > 32 && static_cast<size_t>(dec.F) * (tc + 1) * 4 > 200 * 1024) tc >>= 1;
+  const size_t smem = static_cast<size_t>(dec.F) * (tc + 1) * 4;
   cudaError_t e = cudaFuncSetAttribute(k_decode_rows, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;

@@ -147,16 +147,48 @@ __device__ __forceinline__ float ilog2_exact(float a) {
 
 // One decoded candidate -> column c of the tile (mixed-radix digits, knob 0
 // least significant; then the feature program, one rounded op each).
+// Mixed-radix digit j of candidate idx for every j (knob 0 least
+// significant): 32-bit divisions while the index fits 32 bits (a 64-bit
+// division is a long subroutine), 64-bit ones otherwise.
+__device__ __forceinline__ void knob_digits(const DecodeParams& d, long long idx, int* digit) {
+  if ((static_cast<unsigned long long>(idx) >> 32) == 0) {
+    uint32_t rem = static_cast<uint32_t>(idx);
+    for (int j = 0; j < d.n_knobs; ++j) {
+      const uint32_t r = static_cast<uint32_t>(d.radix[j]);
+      const uint32_t q = rem / r;
+      digit[j] = static_cast<int>(rem - q * r);
+      rem = q;
+    }
+  } else {
+    long long rem = idx;
+    for (int j = 0; j < d.n_knobs; ++j) {
+      const long long r = d.radix[j];
+      const long long q = rem / r;
+      digit[j] = static_cast<int>(rem - q * r);
+      rem = q;
+    }
+  }
+}
+
 __device__ __forceinline__ bool decode_column(const DecodeParams& d, long long idx, float* xs, int TC,
                                               int c) {
   float kv[kMaxKnobs];
-  long long rem = idx;
-  for (int j = 0; j < d.n_knobs; ++j) {
-    const long long r = d.radix[j];
-    const long long q = rem / r;
-    const int digit = static_cast<int>(rem - q * r);
-    rem = q;
-    kv[j] = d.opts[d.opt_off[j] + digit];
+  if ((static_cast<unsigned long long>(idx) >> 32) == 0) {
+    uint32_t rem = static_cast<uint32_t>(idx);
+    for (int j = 0; j < d.n_knobs; ++j) {
+      const uint32_t r = static_cast<uint32_t>(d.radix[j]);
+      const uint32_t q = rem / r;
+      kv[j] = d.opts[d.opt_off[j] + static_cast<int>(rem - q * r)];
+      rem = q;
+    }
+  } else {
+    long long rem = idx;
+    for (int j = 0; j < d.n_knobs; ++j) {
+      const long long r = d.radix[j];
+      const long long q = rem / r;
+      kv[j] = d.opts[d.opt_off[j] + static_cast<int>(rem - q * r)];
+      rem = q;
+    }
   }
   bool nan = false;
   const int nk = d.n_knobs;
