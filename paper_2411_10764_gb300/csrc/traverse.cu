@@ -64,6 +64,8 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
   int tc = 256 / q;
   if (!ov.threads) {
     while (tc > 32 && (n_eff + tc - 1) / tc < (sms + 3) / 4) tc >>= 1;
+    // wide rows: shrink the tile until it fits with the smallest chunk
+    while (tc > 32 && !fits(smem_of(tc, 1, 2))) tc >>= 1;
   } else {
     tc = ov.threads;
   }

@@ -416,3 +416,19 @@ def test_host_batches_pipeline_matches_oracle():
             _, opf, valid, _ = O.screen_rows(b, w.v, w.p, w.thr, threads=THREADS)
             otk, _ = O.topk(opf, valid, w.k)
             assert np.array_equal(tk, otk)
+
+
+@pytest.mark.parametrize("F,depth,shape", [(1, 6, "full"), (1024, 8, "full"), (1024, 12, "unbalanced"),
+                                           (1, 11, "unbalanced"), (1000, 10, "full")])
+def test_feature_count_extremes(F, depth, shape):
+    """The smallest and largest feature rows (1 and 1,024 fp32 features),
+    with full tables and with the deep-tree (compact) walk."""
+    rng = np.random.default_rng(F + depth)
+    n = 2500
+    x = rng.lognormal(0.0, 1.0, size=(n, F)).astype(np.float32)
+    x[rng.random((n, F)) < 0.05] = np.nan
+    cfg = W.ScreenConfig(98, f"f{F}", n, F, 30, depth, 40, depth, 0.5, 100, None, shape=shape)
+    th = W._QuantileThresholds(x[:2048])
+    w = W.Workload(cfg, n, x, None, 0, W.make_ensemble(cfg, "V", th, 7, split_prob=0.8),
+                   W.make_ensemble(cfg, "P", th, 8, split_prob=0.8), 0.5, 100)
+    assert_parity(gpu_screen(w), oracle_screen(w))
