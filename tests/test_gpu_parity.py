@@ -432,3 +432,18 @@ def test_feature_count_extremes(F, depth, shape):
     w = W.Workload(cfg, n, x, None, 0, W.make_ensemble(cfg, "V", th, 7, split_prob=0.8),
                    W.make_ensemble(cfg, "P", th, 8, split_prob=0.8), 0.5, 100)
     assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+@pytest.mark.parametrize("v_trees,p_trees,depth,shape", [(1, 1, 1, "full"), (1, 3, 14, "unbalanced"),
+                                                         (5000, 3000, 3, "full"), (700, 900, 14, "unbalanced")])
+def test_tree_count_and_depth_extremes(v_trees, p_trees, depth, shape):
+    """Stumps and single trees, thousands of shallow trees (many chunks), and
+    the deepest ensembles the library takes (depth 14, compact tables)."""
+    rng = np.random.default_rng(v_trees + depth)
+    n, F = 3001, 24
+    x = rng.lognormal(0.0, 1.0, size=(n, F)).astype(np.float32)
+    cfg = W.ScreenConfig(99, "trees", n, F, v_trees, depth, p_trees, depth, 0.5, n, None, shape=shape)
+    th = W._QuantileThresholds(x[:2048])
+    w = W.Workload(cfg, n, x, None, 0, W.make_ensemble(cfg, "V", th, 3, split_prob=0.8),
+                   W.make_ensemble(cfg, "P", th, 4, split_prob=0.8), 0.5, n)  # k = n: the whole order
+    assert_parity(gpu_screen(w), oracle_screen(w))
