@@ -305,6 +305,14 @@ int mlt_screen_decoded(void *stream, const int32_t *radices, const float *option
  * device (MLT_ETIMEOUT for a bounded wait that gave up), clearing them. */
 int mlt_sync_status(void *stream);
 
+/* Failure-detection self-test: launches one CTA on `stream` that waits on
+ * a shared-memory barrier nothing completes.  The bounded wait every walk
+ * kernel uses gives up after limit_ns (1e6 .. 2e9 ns), records the
+ * timeout and returns, so the next mlt_sync_status(stream) reports
+ * MLT_ETIMEOUT and the device stays usable.  No fault, trap or endless
+ * loop is involved.  Asynchronous. */
+int mlt_selftest_wait_timeout(void *stream, int64_t limit_ns);
+
 /* Number of valid candidates found by the last screening call (waits for
  * `stream`). */
 int mlt_last_survivor_count(void *stream, int64_t *count_out);

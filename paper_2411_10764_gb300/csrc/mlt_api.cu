@@ -1138,6 +1138,19 @@ int mlt_sync_status(void* stream) {
   return fail(MLT_ECUDA, "device-side bookkeeping error (error word 0x%x)", word);
 }
 
+int mlt_selftest_wait_timeout(void* stream, int64_t limit_ns) {
+  if (limit_ns < 1000000LL || limit_ns > static_cast<int64_t>(kWaitLimitNs))
+    return fail(MLT_EINVAL, "limit_ns must lie in [1e6, %llu]", kWaitLimitNs);
+  std::lock_guard<std::mutex> lk(g_mu);
+  const int rc = ensure_scratch(0);  // the device error word
+  if (rc != MLT_OK) return rc;
+  MLT_CUDA(launch_wait_selftest(g_scr.err, static_cast<unsigned long long>(limit_ns),
+                                static_cast<cudaStream_t>(stream)),
+           "self-test launch");
+  g_launches += 1;
+  return MLT_OK;
+}
+
 int mlt_last_survivor_count(void* stream, int64_t* count_out) {
   if (count_out == nullptr) return fail(MLT_EINVAL, "count_out must be non-NULL");
   MLT_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream synchronize");

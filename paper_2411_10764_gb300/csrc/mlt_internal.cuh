@@ -319,6 +319,9 @@ cudaError_t launch_sa_accept(long long space, const int64_t* parent, const float
                              float temperature, int64_t* out_next, float* out_next_score,
                              int32_t* out_accepted, cudaStream_t st);
 
+// selftest.cu: a bounded wait that runs out (failure-detection self-test)
+cudaError_t launch_wait_selftest(unsigned* err, unsigned long long limit_ns, cudaStream_t st);
+
 // rerank.cu
 cudaError_t launch_rerank(const DeviceModel& A, const float* feats, int F, long long n,
                           const int64_t* cand, int m, int n_final, float* out_score,

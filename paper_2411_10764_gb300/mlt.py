@@ -59,6 +59,7 @@ def lib(build_if_missing: bool = True):
             "mlt_load_ensemble": [i32, P, i32, i32],
             "mlt_load_ensemble_f16": [i32, P, i32, i32],
             "mlt_screen_host_batches": [P, i64, P, i64, f32, i32, P, P, P],
+            "mlt_selftest_wait_timeout": [P, i64],
             "mlt_free_ensemble": [i32],
             "mlt_validity_cut": [f32, P],
             "mlt_screen": [P, P, i64, f32, i32, P, P, P],
@@ -335,6 +336,12 @@ def screen_decoded(radices, option_values, program, first_index: int, n: int, th
 
 def sync_status(stream=None) -> None:
     _check(lib().mlt_sync_status(_stream_ptr(stream)))
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
+    """Launch the failure-detection self-test (a device wait that runs out);
+    the next sync_status raises MltError with MLT_ETIMEOUT."""
+    _check(lib().mlt_selftest_wait_timeout(_stream_ptr(stream), int(limit_ns)))
 
 
 def last_survivor_count(stream=None) -> int:

@@ -163,3 +163,9 @@ def test_half_table_loader_rejects(case):
     with pytest.raises(mlt.MltError) as e:
         mlt.load_ensemble_f16(model, nodes, n_trees, depth)
     assert e.value.code == -1
+
+
+@pytest.mark.parametrize("limit", [0, 999_999, 2_000_000_001])
+def test_wait_selftest_rejects_limits(L, limit):
+    # rejected on the host, before any CUDA call
+    assert L.mlt_selftest_wait_timeout(None, limit) == -1
