@@ -113,3 +113,43 @@ def test_half_tables_reject_decoded_screening():
     mlt.load_workload_models(w)  # fp32 tables work again
     mlt.screen_decoded(d.radices, d.option_values, d.program, 0, 1000, w.thr, w.k)
     mlt.sync_status()
+
+
+def test_half_tables_through_the_other_entry_points():
+    """Half tables behind the batched accumulation, the pipelined host
+    batches and the allocation-free entry point: each equals the rounded
+    model's oracle."""
+    import ctypes as C
+
+    import torch
+
+    w = W.make_workload(2, seed=11, n=12000)
+    mlt.load_workload_models(w, half=True)
+    x = O.round_half(w.feats)
+    vh, ph = O.half_ensemble(w.v), O.half_ensemble(w.p)
+    opv, opf, valid, _ = O.screen_rows(x, vh, ph, w.thr, threads=THREADS)
+    otk, s = O.topk(opf, valid, w.k)
+    # batched accumulation over the whole batch (target never reached)
+    _, pf, tk, stats = mlt.screen_until(torch.from_numpy(w.feats).cuda(), 4096, 10 ** 9, w.thr, w.k)
+    mlt.sync_status()
+    assert stats.cpu().tolist()[0] == w.n
+    assert np.array_equal(tk.cpu().numpy(), otk)
+    assert np.array_equal(pf.cpu().numpy().view(np.uint32), opf.view(np.uint32))
+    # pipelined host batches
+    pinned = torch.from_numpy(w.feats).pin_memory().numpy()
+    (pv_h, pf_h, tk_h), = mlt.screen_host_batches([pinned], w.thr, w.k)
+    assert_parity((pv_h, pf_h, tk_h, s), (opv, opf, otk, s))
+    # allocation-free entry point
+    L = mlt.lib()
+    dx = torch.from_numpy(w.feats).cuda()
+    pv2 = torch.empty(w.n, device="cuda")
+    pf2 = torch.empty(w.n, device="cuda")
+    tk2 = torch.empty(w.k, dtype=torch.int64, device="cuda")
+    st = torch.cuda.current_stream()
+    rc = L.mlt_screen_noalloc(C.c_void_p(st.cuda_stream), C.c_void_p(dx.data_ptr()), C.c_int64(w.n), C.c_float(w.thr),
+                              C.c_int(w.k), C.c_void_p(pv2.data_ptr()), C.c_void_p(pf2.data_ptr()),
+                              C.c_void_p(tk2.data_ptr()))
+    assert rc == 0
+    mlt.sync_status()
+    assert_parity((pv2.cpu().numpy(), pf2.cpu().numpy(), tk2.cpu().numpy(), s), (opv, opf, otk, s))
+    mlt.load_workload_models(w)
