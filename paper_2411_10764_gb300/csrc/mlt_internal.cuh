@@ -222,6 +222,7 @@ struct ScreenShape {
   int lanes = 1;       // threads sharing one candidate's trees: warp groups (full tables) or
                        // lanes of a warp (compact tables); CTA = threads * lanes
   int p_grid = 0;      // full-table P pass: CTAs one wave holds (resident per SM x SMs)
+  int sync_free = 0;   // full tables, one tree group: barrier-free chunk pipeline (one CTA per SM)
   int resident = 0;    // full tables: CTAs meant to share an SM (shared memory is padded so
                        // that no more fit: the block scheduler would otherwise stack tiles
                        // on some SMs and leave others idle)
@@ -241,6 +242,8 @@ struct ShapeOverride {
 // traverse_q2.cu (Q = 2), traverse_q4.cu (Q = 4).  nullptr if not built.
 using FullKernelPtr = void (*)(TraverseArgs);
 using FullDecKernelPtr = void (*)(TraverseArgs, DecodeParams);
+// q = tree groups (1, 2, 4), or 0 for one group with the barrier-free
+// chunk pipeline
 FullKernelPtr full_kernel(int depth, int group, int q);
 FullDecKernelPtr full_dec_kernel(int depth, int group, int q);
 FullKernelPtr full_kernel_q1(int depth, int group);
@@ -249,8 +252,11 @@ FullKernelPtr full_kernel_q2(int depth, int group);
 FullDecKernelPtr full_dec_kernel_q2(int depth, int group);
 FullKernelPtr full_kernel_q4(int depth, int group);
 FullDecKernelPtr full_dec_kernel_q4(int depth, int group);
+// traverse_sf.cu: one tree group, barrier-free chunk pipeline
+FullKernelPtr full_kernel_sf(int depth, int group);
+FullDecKernelPtr full_dec_kernel_sf(int depth, int group);
 // traverse_half.cu: half tables (one tree group, stored features only)
-FullKernelPtr half_kernel(int depth, int group);
+FullKernelPtr half_kernel(int depth, int group, bool sync_free);
 
 // traverse.cu
 // n_eff: candidates the pass is expected to walk (used for load balance).

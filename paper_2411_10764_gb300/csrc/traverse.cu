@@ -21,6 +21,7 @@ FullKernelPtr full_kernel_q1(int depth, int group) { return full_kernel_q<1>(dep
 
 FullKernelPtr full_kernel(int depth, int group, int q) {
   switch (q) {
+    case 0: return full_kernel_sf(depth, group);
     case 1: return full_kernel_q1(depth, group);
     case 2: return full_kernel_q2(depth, group);
     case 4: return full_kernel_q4(depth, group);
@@ -102,6 +103,7 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
         best.smem = smem;
         best.p_grid = sms * std::max(1, res);  // CTAs per wave: the tiles an SM gets, up to residency
         best.resident = std::max(1, res);
+        best.sync_free = q == 1 && best.resident == 1 ? 1 : 0;
       }
     }
   }
@@ -224,8 +226,9 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
   }
   const dim3 grid(static_cast<unsigned>(ctas));
   if (m.kind != kTableCompact) {
-    FullKernelPtr k = m.kind == kTableHalf ? (shape.lanes == 1 ? half_kernel(m.depth, shape.group) : nullptr)
-                                           : full_kernel(m.depth, shape.group, shape.lanes);
+    FullKernelPtr k = m.kind == kTableHalf
+                          ? (shape.lanes == 1 ? half_kernel(m.depth, shape.group, shape.sync_free != 0) : nullptr)
+                          : full_kernel(m.depth, shape.group, shape.sync_free ? 0 : shape.lanes);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));

@@ -79,6 +79,7 @@ FullDecKernelPtr full_dec_kernel_q1(int depth, int group) { return full_dec_kern
 
 FullDecKernelPtr full_dec_kernel(int depth, int group, int q) {
   switch (q) {
+    case 0: return full_dec_kernel_sf(depth, group);
     case 1: return full_dec_kernel_q1(depth, group);
     case 2: return full_dec_kernel_q2(depth, group);
     case 4: return full_dec_kernel_q4(depth, group);
@@ -100,7 +101,7 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
   }
   const dim3 grid(static_cast<unsigned>(ctas));
   if (m.kind == kTableFull) {
-    FullDecKernelPtr k = full_dec_kernel(m.depth, shape.group, shape.lanes);
+    FullDecKernelPtr k = full_dec_kernel(m.depth, shape.group, shape.sync_free ? 0 : shape.lanes);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));

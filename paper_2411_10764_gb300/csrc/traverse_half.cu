@@ -5,10 +5,15 @@
 
 namespace mlt {
 
-FullKernelPtr half_kernel(int depth, int group) {
-  return group == 8   ? walk::half_kernel_for<8>(depth)
-         : group == 4 ? walk::half_kernel_for<4>(depth)
-         : group == 2 ? walk::half_kernel_for<2>(depth)
+FullKernelPtr half_kernel(int depth, int group, bool sync_free) {
+  if (sync_free)
+    return group == 8   ? walk::half_kernel_for<8, 0>(depth)
+           : group == 4 ? walk::half_kernel_for<4, 0>(depth)
+           : group == 2 ? walk::half_kernel_for<2, 0>(depth)
+                        : nullptr;
+  return group == 8   ? walk::half_kernel_for<8, 1>(depth)
+         : group == 4 ? walk::half_kernel_for<4, 1>(depth)
+         : group == 2 ? walk::half_kernel_for<2, 1>(depth)
                       : nullptr;
 }
 

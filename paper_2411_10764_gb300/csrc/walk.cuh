@@ -671,8 +671,15 @@ __device__ __forceinline__ void cta_tile(const TraverseArgs& a, long long count,
 // order one chunk later (two leaf buffers), so the sum is the same
 // sequential fp32 sum as with one walker.  More groups put more warps on a
 // small batch; all lanes of a warp still walk the same tree.
-template <int D, int G, int Q, bool H = false>
+// QS = tree groups, or 0 for one group with the barrier-free chunk
+// pipeline: each warp counts itself out of a chunk buffer and the last one
+// refills it, so warps drift up to nbuf - 1 chunks apart instead of meeting
+// at a CTA barrier per chunk.  That wins where one CTA holds the SM; with two
+// resident CTAs the barrier version keeps the refills further ahead.
+template <int D, int G, int QS, bool H = false>
 __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
+  constexpr int Q = QS == 0 ? 1 : QS;
+  constexpr bool kSyncFree = QS == 0;
   static_assert(!H || Q == 1, "half tables walk with one tree group");
   constexpr int xb = H ? 2 : 4;  // bytes per staged feature
   extern __shared__ __align__(128) unsigned char smem[];
@@ -699,9 +706,17 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   unsigned long long* bars = reinterpret_cast<unsigned long long*>(
       smem + leaf_off + full_smem_leaf_bytes(TC, Q, a.chunk_trees));
   const int n_chunks = (a.n_trees + a.chunk_trees - 1) / a.chunk_trees;
+  // barrier-free pipeline: warps release a chunk buffer by counting
+  // themselves out; the last one refills it
+  __shared__ unsigned released[4];
+  __shared__ int last_issued[4];  // latest chunk copied into each buffer
 
   if (tid == 0) {
     for (int b = 0; b < a.nbuf; ++b) mbar_init(smem_u32(&bars[b]), 1);
+    for (int b = 0; b < 4; ++b) {
+      released[b] = 0u;
+      last_issued[b] = b < n_chunks ? b : -1;
+    }
     fence_mbar_init();
   }
   __syncthreads();
@@ -738,6 +753,49 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   // parked leaves: buffer p holds leaf t of candidate c at la[p] + t * row_bytes
   const uint32_t la0 = smem_u32(smem + leaf_off) + static_cast<uint32_t>(c) * 4u;
   const uint32_t la_step = static_cast<uint32_t>(a.chunk_trees) * row_bytes;
+  if constexpr (kSyncFree) {
+    const int n_warps = static_cast<int>(blockDim.x >> 5);
+    const int lane = tid & 31;
+    bool timed_out = false;
+    for (int ch = 0; ch < n_chunks; ++ch) {
+      const int b = ch % a.nbuf;
+      const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
+      if (!__all_sync(0xFFFFFFFFu, ok)) {
+        timed_out = true;
+        break;
+      }
+      const uint32_t tb = tbuf_a + static_cast<uint32_t>(b) * chunk_bytes;
+      const int nt = min(a.chunk_trees, a.n_trees - ch * a.chunk_trees);
+      if constexpr (H)
+        acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
+                  : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+      else
+        acc = nan ? walk_chunk<D, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u)
+                  : walk_chunk<D, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u);
+      __syncwarp();
+      if (lane == 0 && ch + a.nbuf < n_chunks) {
+        __threadfence_block();  // this warp's reads of buffer b are done
+        if (atomicAdd(&released[b], 1u) == static_cast<unsigned>(n_warps - 1)) {
+          released[b] = 0u;
+          last_issued[b] = ch + a.nbuf;
+          __threadfence_block();
+          issue(ch + a.nbuf, b);  // the last warp out refills it
+        }
+      }
+    }
+    if (__syncthreads_or(timed_out)) {
+      if (tid == 0) {
+        // the copy last issued into each buffer lands before the CTA's
+        // shared memory is released (bounded waits), then the timeout is
+        // reported
+        for (int b = 0; b < a.nbuf; ++b)
+          if (last_issued[b] >= 0)
+            mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(last_issued[b] / a.nbuf) & 1u);
+        atomicOr(a.err, kErrWaitTimeout);
+      }
+      return;
+    }
+  } else
   for (int ch = 0; ch < n_chunks; ++ch) {
     const int b = ch % a.nbuf;
     const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
@@ -790,24 +848,24 @@ __global__ void __launch_bounds__(256)
   traverse_full_body<D, G, Q>(a, &d);
 }
 
-template <int D, int G>
+template <int D, int G, int QS>
 __global__ void __launch_bounds__(256) k_traverse_half(const __grid_constant__ TraverseArgs a) {
-  traverse_full_body<D, G, 1, true>(a, nullptr);
+  traverse_full_body<D, G, QS, true>(a, nullptr);
 }
 
-template <int G>
+template <int G, int QS>
 FullKernelPtr half_kernel_for(int d) {
   switch (d) {
-    case 1: return k_traverse_half<1, G>;
-    case 2: return k_traverse_half<2, G>;
-    case 3: return k_traverse_half<3, G>;
-    case 4: return k_traverse_half<4, G>;
-    case 5: return k_traverse_half<5, G>;
-    case 6: return k_traverse_half<6, G>;
-    case 7: return k_traverse_half<7, G>;
-    case 8: return k_traverse_half<8, G>;
-    case 9: return k_traverse_half<9, G>;
-    case 10: return k_traverse_half<10, G>;
+    case 1: return k_traverse_half<1, G, QS>;
+    case 2: return k_traverse_half<2, G, QS>;
+    case 3: return k_traverse_half<3, G, QS>;
+    case 4: return k_traverse_half<4, G, QS>;
+    case 5: return k_traverse_half<5, G, QS>;
+    case 6: return k_traverse_half<6, G, QS>;
+    case 7: return k_traverse_half<7, G, QS>;
+    case 8: return k_traverse_half<8, G, QS>;
+    case 9: return k_traverse_half<9, G, QS>;
+    case 10: return k_traverse_half<10, G, QS>;
     default: return nullptr;
   }
 }
@@ -847,7 +905,8 @@ FullDecKernelPtr full_dec_kernel_for(int d) {
   }
 }
 
-// All depths and G in {2, 4, 8} for one Q (each Q is instantiated in its own
+// All depths and G in {2, 4, 8} for one QS (tree groups, or 0 for one group
+// with the barrier-free pipeline; each QS is instantiated in its own
 // translation unit, compiled in parallel).
 template <int Q>
 FullKernelPtr full_kernel_q(int d, int g) {
