@@ -273,10 +273,7 @@ ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeO
                       : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
   if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
     return plan_for(dm, F, n_eff, ShapeOverride(), v_pass);
-  // the P pass splits its survivors evenly over the CTAs on the device, so
-  // its CTA size is balanced for the estimate as well
-  if (dm.kind != kTableCompact && ov.threads == 0)
-    s = balance_full_tiles(s, F, dm.tree_bytes, n_eff, sm_count(), half);
+  // no more CTAs per SM than the plan counted on
   if (dm.kind != kTableCompact) s = cap_residency(s, smem_optin());
   return s;
 }

@@ -265,10 +265,6 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, 
                       int device_smem_optin, const ShapeOverride& ov, bool half);
 ScreenShape plan_compact(int F, long long n_eff, int sms, int device_smem_optin,
                          const ShapeOverride& ov);
-// V pass over n known candidates: the smallest multiple of 32 candidates
-// per CTA (at least 64) that leaves the busiest SM no more tiles than `s`
-// does, so the tiles spread evenly over the SMs.
-ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms, bool half);
 // Pad a full-table shape's shared memory so that at most s.resident CTAs fit
 // on an SM.
 ScreenShape cap_residency(const ScreenShape& s, int optin);

@@ -40,8 +40,8 @@ FullKernelPtr full_kernel(int depth, int group, int q) {
 //     CTAs resident (twice the warps to hide shared-memory latency) beats
 //     one CTA with bigger chunks: take the largest chunk that still allows
 //     two; otherwise one CTA with the largest chunk (fewest barriers);
-//   * a thread walks 8 trees at once when 8 warps or fewer share the SM,
-//     else 4 (the chunk permitting);
+//   * a thread walks 8 trees at once (4 with tree groups when more than 8
+//     warps share the SM), the chunk permitting;
 //   * a batch of under 32 (64) candidates per SM splits each tile's trees
 //     over 4 (2) groups of warps.
 ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms, int optin,
@@ -67,6 +67,13 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
     while (tc > 32 && (n_eff + tc - 1) / tc < (sms + 3) / 4) tc >>= 1;
     // wide rows: shrink the tile until it fits with the smallest chunk
     while (tc > 32 && !fits(smem_of(tc, 1, 2))) tc >>= 1;
+    // spread the tiles evenly: the smallest multiple of 32 (at least 64)
+    // that gives the busiest SM no more tiles; decided before the chunk
+    // size, which the smaller tile may let grow
+    const long long t_sm = ((n_eff + tc - 1) / tc + sms - 1) / sms;
+    const long long per_tile = (n_eff + sms * t_sm - 1) / (sms * t_sm);
+    const int tb = static_cast<int>(std::min<long long>(tc, (per_tile + 31) / 32 * 32));
+    if (tb >= 64) tc = tb;
   } else {
     tc = ov.threads;
   }
@@ -90,7 +97,7 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
       if (rank > best_rank) {
         best_rank = rank;
         const int warps = res * tc * q / 32;
-        int group = warps <= 8 ? 8 : 4;
+        int group = q == 1 || warps <= 8 ? 8 : 4;
         if (ov.group) group = ov.group;
         // each group walks chunk / q trees of a chunk
         const int per = std::max(1, chunk / q);
@@ -108,20 +115,6 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
     }
   }
   return best;  // threads == 0: nothing fits
-}
-
-ScreenShape balance_full_tiles(const ScreenShape& s, int F, uint32_t tree_bytes, long long n, int sms, bool half) {
-  if (s.threads == 0 || n <= 0 || sms < 1) return s;
-  const long long tiles_sm = ((n + s.threads - 1) / s.threads + sms - 1) / sms;
-  const long long per_tile = (n + sms * tiles_sm - 1) / (sms * tiles_sm);
-  const int tc = static_cast<int>(std::min<long long>(s.threads, std::max<long long>(32, (per_tile + 31) / 32 * 32)));
-  // below two warps per CTA the table stream, not the walk, sets the pace
-  if (tc < 64 || tc == s.threads) return s;
-  ScreenShape b = s;
-  b.threads = tc;
-  b.smem = full_smem_bytes(F, tc, s.nbuf, static_cast<uint32_t>(s.chunk_trees) * tree_bytes, s.lanes,
-                           s.chunk_trees, half ? 2 : 4);
-  return b;
 }
 
 ScreenShape cap_residency(const ScreenShape& s, int optin) {
