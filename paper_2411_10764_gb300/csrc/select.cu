@@ -11,17 +11,20 @@
 // largest keys" is exactly "k best by (score desc, position asc)"; it also
 // counts the keys' top 12 bits in a histogram.  One top-k kernel then finds
 // the histogram bucket holding the k-th key, collects every key in that
-// bucket or above (a few thousand for the workloads here), and the last CTA
-// to finish (ticket counter, no waiting) sorts them in shared memory.  If
-// ties crowd more keys into the collection than shared memory holds, that
-// CTA first narrows them with an exact most-significant-digit radix select.
+// bucket or above (a few hundred to a few thousand for the workloads here),
+// and the last CTA to finish (ticket counter, no waiting) narrows them to
+// exactly the k best with an exact most-significant-digit radix select
+// (8-bit digits below the bucket's bits, counted in shared memory) and
+// orders those: by counting for each key the larger ones (up to 512 keys),
+// else by a bitonic sort.
 #include "mlt_internal.cuh"
 
 namespace mlt {
 namespace {
 
 constexpr int kTopkThreads = 512;
-constexpr int kSortMin = 8192;  // sort buffer entries (at least pow2(k))
+constexpr int kSortMin = 8192;  // collected keys held in shared memory
+constexpr unsigned kRankMax = 512;  // order by rank counting up to this many keys
 
 __global__ void __launch_bounds__(256)
     k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n, const StreamState* ss) {
@@ -60,12 +63,32 @@ __device__ void sort_desc(unsigned long long* sk, int n2) {
   }
 }
 
+// Rank of every key among out_keys[0, kk) (keys unique), by counting the
+// larger ones: no barrier, cheaper than a bitonic sort for a few hundred
+// keys.  out_keys[kk] must be readable (0 when kk is odd: smaller than any key).
+__device__ void write_by_rank(const unsigned long long* out_keys, unsigned kk, long long base, int64_t* out) {
+  const ulonglong2* pairs = reinterpret_cast<const ulonglong2*>(out_keys);
+  const unsigned n_pairs = (kk + 1u) >> 1;
+  for (unsigned i = threadIdx.x; i < kk; i += blockDim.x) {
+    const unsigned long long key = out_keys[i];
+    unsigned r = 0;
+    for (unsigned j = 0; j < n_pairs; ++j) {
+      const ulonglong2 q = pairs[j];
+      r += (q.x > key) + (q.y > key);
+    }
+    const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull);
+    out[r] = base + static_cast<long long>(pos);
+  }
+}
+
 __global__ void __launch_bounds__(kTopkThreads)
-    k_topk(const unsigned long long* keys, unsigned long long* cand, SelectState* st, int k, int cap,
+    k_topk(const unsigned long long* keys, unsigned long long* cand, SelectState* st, int k, int n2k,
            long long base, int64_t* out, unsigned* err, const unsigned* count) {
-  extern __shared__ __align__(16) unsigned long long sk[];  // cap entries
+  // sk[0, kSortMin): the collected keys when they fit; sk[kSortMin, +n2k):
+  // the kk selected keys (n2k = pow2 >= k, at least 2)
+  extern __shared__ __align__(16) unsigned long long sk[];
   __shared__ unsigned warp_sum[kTopkThreads / 32];
-  __shared__ unsigned s_bin, s_last, s_digit, s_rem, s_h, s_cnt;
+  __shared__ unsigned s_bin, s_above, s_hbin, s_last, s_digit, s_rem, s_h, s_cnt;
   __shared__ unsigned h256[256];
   pdl_wait();
   const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -96,7 +119,11 @@ __global__ void __launch_bounds__(kTopkThreads)
   for (int w = 0; w < warp; ++w) above += warp_sum[w];
 #pragma unroll
   for (int q = 0; q < per; ++q) {
-    if (kk > 0 && above < kk && kk <= above + hb[q]) s_bin = static_cast<unsigned>(kTopBins - 1 - (tid * per + q));
+    if (kk > 0 && above < kk && kk <= above + hb[q]) {
+      s_bin = static_cast<unsigned>(kTopBins - 1 - (tid * per + q));
+      s_above = above;
+      s_hbin = hb[q];
+    }
     above += hb[q];
   }
   __syncthreads();
@@ -121,7 +148,9 @@ __global__ void __launch_bounds__(kTopkThreads)
     }
   }
 
-  // 3. the last CTA to finish selects and sorts
+  // 3. the last CTA to finish narrows the collection to exactly the kk best
+  //    keys (8-bit digits below the bucket's 12 bits, counted in shared
+  //    memory) and orders them
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
@@ -130,74 +159,85 @@ __global__ void __launch_bounds__(kTopkThreads)
   __threadfence();
   const unsigned m = *reinterpret_cast<volatile unsigned*>(&st->n_cand);
   if (tid == 0) st->v_ticket = 0u;  // in case a V pass ended early
-  int n2 = 1;
-  while (n2 < static_cast<int>(kk)) n2 <<= 1;
-  if (m <= static_cast<unsigned>(cap)) {
-    // every collected key fits: sort them all, keep the first kk
-    int m2 = 1;
-    while (m2 < static_cast<int>(m)) m2 <<= 1;
-    for (int i = tid; i < m2; i += T) sk[i] = i < static_cast<int>(m) ? __ldcg(cand + i) : 0ull;
+  unsigned long long* out_keys = sk + kSortMin;
+  if (kk > 0) {
+    const bool in_smem = m <= static_cast<unsigned>(kSortMin);
+    if (in_smem)
+      for (unsigned i = tid; i < m; i += T) sk[i] = __ldcg(cand + i);
+    auto key_at = [&](unsigned i) { return in_smem ? sk[i] : __ldcg(cand + i); };
+    unsigned long long mask = ~0ull << (64 - kTopBits);
+    unsigned long long prefix = bin << (64 - kTopBits);
+    unsigned rem = kk - s_above;  // keys of the boundary bucket still wanted
+    bool finished = s_hbin == rem;
     __syncthreads();
-    sort_desc(sk, m2);
-  } else {
-    // heavy ties: exact radix select of the kk-th key among the collected
-    // keys (8-bit digits from the top), then gather the kk keys above it
-    unsigned long long prefix = 0, mask = 0;
-    unsigned rem = kk;
-    for (int shift = 56; shift >= 0; shift -= 8) {
-      for (int i = tid; i < 256; i += T) h256[i] = 0u;
+    for (int hi = 64 - kTopBits; hi > 0 && !finished; hi -= 8) {
+      const int shift = hi > 8 ? hi - 8 : 0;
+      const unsigned long long dmask = (1ull << (hi - shift)) - 1ull;
+      if (tid < 256) h256[tid] = 0u;
       __syncthreads();
       for (unsigned i = tid; i < m; i += T) {
-        const unsigned long long key = __ldcg(cand + i);
-        if ((key & mask) == prefix) atomicAdd(&h256[(key >> shift) & 0xFFull], 1u);
+        const unsigned long long key = key_at(i);
+        if ((key & mask) == prefix) atomicAdd(&h256[(key >> shift) & dmask], 1u);
       }
       __syncthreads();
-      if (tid == 0) {
-        unsigned cum = 0;
-        for (int d = 255; d >= 0; --d) {
-          const unsigned h = h256[d];
-          if (cum + h >= rem) {
-            s_digit = static_cast<unsigned>(d);
-            s_rem = rem - cum;
-            s_h = h;
-            break;
-          }
-          cum += h;
+      // digit of the rem-th key: scan the 256 counts from the top digit down
+      unsigned h = 0, incl = 0;
+      if (tid < 256) {
+        h = h256[255 - tid];
+        incl = h;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (lane == 31) warp_sum[warp] = incl;
+      }
+      __syncthreads();
+      if (tid < 256) {
+        unsigned ab = incl - h;
+        for (int w = 0; w < warp; ++w) ab += warp_sum[w];
+        if (ab < rem && rem <= ab + h) {
+          s_digit = static_cast<unsigned>(255 - tid);
+          s_rem = rem - ab;
+          s_h = h;
         }
       }
       __syncthreads();
       prefix |= static_cast<unsigned long long>(s_digit) << shift;
-      mask |= 0xFFull << shift;
+      mask |= dmask << shift;
       rem = s_rem;
-      const bool finished = s_h == rem;
-      __syncthreads();
-      if (finished) break;
+      finished = s_h == rem;
+      __syncthreads();  // s_* and h256 are rewritten by the next digit
     }
     if (tid == 0) s_cnt = 0u;
     __syncthreads();
     for (unsigned i = tid; i < m; i += T) {
-      const unsigned long long key = __ldcg(cand + i);
+      const unsigned long long key = key_at(i);
       if ((key & mask) >= prefix) {
         const unsigned p = atomicAdd(&s_cnt, 1u);
         if (p < kk)
-          sk[p] = key;
+          out_keys[p] = key;
         else
           atomicOr(err, kErrSelect);
       }
     }
+    if (tid == 0 && (kk & 1u)) out_keys[kk] = 0ull;  // pad for the pairwise rank loop (kk odd < n2k)
     __syncthreads();
-    for (int i = static_cast<int>(kk) + tid; i < n2; i += T) sk[i] = 0ull;
-    __syncthreads();
-    sort_desc(sk, n2);
-  }
-  for (int r = tid; r < k; r += T) {
-    if (r < static_cast<int>(kk)) {
-      const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(sk[r] & 0xFFFFFFFFull);
-      out[r] = base + static_cast<long long>(pos);
+    if (kk <= kRankMax) {
+      write_by_rank(out_keys, kk, base, out);
     } else {
-      out[r] = -1;
+      int n2 = 1;
+      while (n2 < static_cast<int>(kk)) n2 <<= 1;
+      for (int i = static_cast<int>(kk) + tid; i < n2; i += T) out_keys[i] = 0ull;
+      __syncthreads();
+      sort_desc(out_keys, n2);
+      for (int r = tid; r < static_cast<int>(kk); r += T) {
+        const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(out_keys[r] & 0xFFFFFFFFull);
+        out[r] = base + static_cast<long long>(pos);
+      }
     }
   }
+  for (int r = static_cast<int>(kk) + tid; r < k; r += T) out[r] = -1;
 }
 
 }  // namespace
@@ -247,16 +287,16 @@ cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaS
 
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk, int sms,
                         const unsigned* count, cudaStream_t st) {
-  int cap = kSortMin;
-  while (cap < k) cap <<= 1;
-  const size_t smem = static_cast<size_t>(cap) * 8;
+  int n2k = 2;
+  while (n2k < k) n2k <<= 1;
+  const size_t smem = static_cast<size_t>(kSortMin + n2k) * 8;
   cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   long long g = (n + 1023) / 1024;  // about one pass of the collection loop per warp
   if (g < 1) g = 1;
   if (g > 4LL * sms) g = 4LL * sms;
   return launch_pdl(k_topk, dim3(static_cast<unsigned>(g)), dim3(kTopkThreads), smem, st,
-                    static_cast<const unsigned long long*>(s.keys), s.cand, s.state, k, cap, index_base, out_topk,
+                    static_cast<const unsigned long long*>(s.keys), s.cand, s.state, k, n2k, index_base, out_topk,
                     s.err, count);
 }
 

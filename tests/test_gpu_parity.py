@@ -59,6 +59,39 @@ def test_k_sizes_including_more_than_survivors(k):
     assert_parity(gpu_screen(w, k=k), oracle_screen(w, k=k))
 
 
+@pytest.fixture(scope="module")
+def mid():
+    w = W.make_workload(2, seed=4, n=20000)
+    return w, oracle_screen(w, k=8000)
+
+
+@pytest.mark.parametrize("k", [2, 63, 300, 511, 512, 513, 1000, 4099])
+def test_k_sizes_around_the_ordering_switch(mid, k):
+    """Up to 512 selected keys are ordered by counting, more by a sort."""
+    w, (opv, opf, otk, os_) = mid
+    assert_parity(gpu_screen(w, k=k), (opv, opf, otk[:k], os_))
+
+
+@pytest.fixture(scope="module")
+def all_tied():
+    """30,000 copies of one surviving candidate: every key shares its score,
+    so the whole collection (more than shared memory holds) sits in the
+    boundary bucket and the selection runs down to the position digits."""
+    w = W.make_workload(2, seed=1, n=2000)
+    _, _, valid, _ = O.screen_rows(w.feats, w.v, w.p, w.thr, threads=THREADS)
+    row = w.feats[int(np.nonzero(valid)[0][0])]
+    x = np.ascontiguousarray(np.tile(row, (30000, 1)))
+    return w, x, oracle_screen(w, feats=x, k=16384)
+
+
+@pytest.mark.parametrize("k", [1, 100, 512, 513, 4096, 16384])
+def test_topk_when_every_score_ties(all_tied, k):
+    w, x, (opv, opf, otk, os_) = all_tied
+    assert os_ == 30000
+    assert np.array_equal(otk[:k], np.arange(k))
+    assert_parity(gpu_screen(w, feats=x, k=k), (opv, opf, otk[:k], os_))
+
+
 @pytest.mark.parametrize("thr", [1e-6, 0.999999, 0.3, 0.75])
 def test_thresholds_all_none_some(thr):
     w = W.make_workload(1, seed=1, n=4096)
