@@ -191,13 +191,16 @@ def config_dict(w):
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
-def library_source_hash() -> str:
-    """Hash of the CUDA sources and the C header (order as in the profiles)."""
+def walk_source_hash() -> str:
+    """Hash of the sources the tree-walk kernels compile from (the walk
+    device code, the launch planners and instantiations, the internal header
+    and the C header), in a fixed order."""
     import glob
     import hashlib
 
     csrc = os.path.join(ROOT, "paper_2411_10764_gb300", "csrc")
-    files = sorted(glob.glob(os.path.join(csrc, "*.cu"))) + sorted(glob.glob(os.path.join(csrc, "*.cuh")))
+    files = [os.path.join(csrc, "walk.cuh"), os.path.join(csrc, "mlt_internal.cuh")]
+    files += sorted(glob.glob(os.path.join(csrc, "traverse*.cu")))
     files.append(os.path.join(ROOT, "include", "mlt.h"))
     h = hashlib.sha256()
     for path in files:
@@ -207,15 +210,15 @@ def library_source_hash() -> str:
 
 
 def dram_traffic(config: int, phase: str):
-    """DRAM bytes per launch of the phase's kernel from the committed ncu
-    capture, or None if there is none or the kernels changed since."""
+    """DRAM bytes per launch of the phase's walk kernel from the committed
+    ncu capture, or None if there is none or the walk sources changed since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             tr = json.load(f)
     except (OSError, ValueError):
         return None
-    if tr.get("source_hash") != library_source_hash():
+    if tr.get("walk_source_hash") != walk_source_hash():
         return None
     ent = tr.get(f"config{config}:{phase}")
     return ent.get("dram_bytes_per_launch") if ent else None
