@@ -323,6 +323,22 @@ int mlt_last_survivor_count(void *stream, int64_t *count_out);
  * bookkeeping plus event records; results are unchanged. */
 int mlt_profile_phases(int enable);
 
+/* Measurement support: the walk-rate ceiling of a full-table model (depth
+ * <= 10) on this batch.  One launch stages tiles of the candidates
+ * feats[0, n) (device, [n][F] fp32, as for mlt_screen) the way the V pass
+ * does, copies the first R trees of model `model_id`'s table into shared
+ * memory once (R = the trees the V-pass shape keeps in its chunk buffers,
+ * at most the model's), and walks those R trees `rounds` times per
+ * candidate: the screening walk's node test and layout without its chunk
+ * streaming.  out_sums[i] (device, [n]) receives the fp32 sum, in walk order,
+ * of the rounds x R leaves candidate i reaches (trees 0..R-1, repeated);
+ * *visits_out receives the node visits of the launch (n x R x depth x
+ * rounds).  The caller times the launch with events on `stream`.
+ * Asynchronous; MLT_EINVAL for a bad argument, a compact table or a half
+ * table; MLT_ENOMODEL if the model is not loaded for the current F. */
+int mlt_walk_peak(void *stream, int model_id, const float *feats, int64_t n, int rounds, float *out_sums,
+                  int64_t *visits_out);
+
 /* Waits for the recorded events, then writes for each phase the device time
  * summed over the recorded calls, in ms: out_ms[0] V pass, [1] survivor
  * compaction, [2] P pass, [3] top-k (n_phases <= 4 entries written).

@@ -22,6 +22,7 @@
 #include <cuda_fp16.h>
 
 #include "mlt_internal.cuh"
+#include "peak.cuh"
 
 // Scratch of mlt_screen_noalloc: one fixed array in the module's global
 // memory (about 5.1 MB, held on every device that loads the library until
@@ -1187,6 +1188,57 @@ int mlt_phase_times(float* out_ms, int n_phases, int64_t* n_calls_out) {
   for (int p = 0; p < n_phases && p < kPhases; ++p) out_ms[p] = static_cast<float>(sum[p]);
   *n_calls_out = static_cast<int64_t>(calls);
   g_events_used = 0;
+  return MLT_OK;
+}
+
+int mlt_walk_peak(void* stream, int model_id, const float* feats, int64_t n, int rounds, float* out_sums,
+                  int64_t* visits_out) {
+  if (model_id != MLT_MODEL_V && model_id != MLT_MODEL_P) return fail(MLT_EINVAL, "model_id must be V or P");
+  if (n < 1 || n > 0x7FFFFFFFLL) return fail(MLT_EINVAL, "n must lie in [1, 2^31-1]");
+  if (rounds < 1 || rounds > 1000000) return fail(MLT_EINVAL, "rounds must lie in [1, 1e6]");
+  if (feats == nullptr || out_sums == nullptr || visits_out == nullptr)
+    return fail(MLT_EINVAL, "feats, out_sums and visits_out must be non-NULL");
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_F <= 0) return fail(MLT_ENOMODEL, "no feature count set");
+  const Model& m = g_models[model_id];
+  if (!m.loaded || m.F != g_F) return fail(MLT_ENOMODEL, "model %d is not loaded for F=%d", model_id, g_F);
+  if (m.dm.kind != kTableFull) return fail(MLT_EINVAL, "the walk-rate ceiling needs a full fp32 table (depth <= %d)", kMaxFullDepth);
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  if (m.device != dev) return fail(MLT_EINVAL, "model %d lives on device %d, current device is %d", model_id, m.device, dev);
+  const DeviceModel& dm = m.dm;
+  const ScreenShape s = plan_for(dm, g_F, n, g_shape[model_id], true);
+  if (s.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
+  // one thread per candidate (a tree-group shape becomes one wider group)
+  const int tc = std::min(256, s.threads * s.lanes);
+  const size_t feat_bytes = walk_peak_tree_offset(g_F, tc);
+  int resident = std::min(dm.n_trees, s.chunk_trees * s.nbuf);
+  while (resident > 1 && feat_bytes + static_cast<size_t>(resident) * dm.tree_bytes + 1024 > static_cast<size_t>(smem_optin()))
+    --resident;
+  const size_t smem = feat_bytes + static_cast<size_t>(resident) * dm.tree_bytes;
+  if (smem + 1024 > static_cast<size_t>(smem_optin())) return fail(MLT_EINVAL, "F=%d leaves no room for a tree", g_F);
+  WalkPeakKernelPtr k = walk_peak_kernel(dm.depth, s.group);
+  if (k == nullptr) return fail(MLT_EINVAL, "no walk-rate kernel for depth %d, group %d", dm.depth, s.group);
+  rc = ensure_scratch(0);  // the device error word
+  if (rc != MLT_OK) return rc;
+  TraverseArgs a{};
+  a.feats = feats;
+  a.F = g_F;
+  a.n = n;
+  a.vec4 = ((reinterpret_cast<uintptr_t>(feats) & 15u) == 0 && (g_F & 3) == 0) ? 1 : 0;
+  a.table = dm.table;
+  a.n_trees = dm.n_trees;
+  a.tree_bytes = dm.tree_bytes;
+  a.err = g_scr.err;
+  MLT_CUDA(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)),
+           "walk-rate kernel attribute");
+  const long long tiles = (n + tc - 1) / tc;
+  k<<<dim3(static_cast<unsigned>(tiles)), dim3(tc), smem, static_cast<cudaStream_t>(stream)>>>(a, resident, rounds,
+                                                                                             out_sums);
+  MLT_CUDA(cudaGetLastError(), "walk-rate kernel launch");
+  g_launches += 1;
+  *visits_out = static_cast<int64_t>(n) * resident * dm.depth * rounds;
   return MLT_OK;
 }
 

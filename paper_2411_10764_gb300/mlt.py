@@ -71,6 +71,7 @@ def lib(build_if_missing: bool = True):
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
+            "mlt_walk_peak": [P, i32, P, i64, i32, P, P],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
             "mlt_screen_until": [P, P, i64, i64, i64, f32, i32, P, P, P, P],
@@ -342,6 +343,26 @@ def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
     """Launch the failure-detection self-test (a device wait that runs out);
     the next sync_status raises MltError with MLT_ETIMEOUT."""
     _check(lib().mlt_selftest_wait_timeout(_stream_ptr(stream), int(limit_ns)))
+
+
+def walk_peak(feats, rounds: int, model_id: int = MLT_MODEL_V, out_sums=None, stream=None):
+    """mlt_walk_peak: walk the first trees of a full-table model, held in
+    shared memory, `rounds` times for every row of `feats` (a [n][F] fp32
+    CUDA tensor).  Returns (sums, visits): the per-row fp32 leaf sums and the
+    node visits of the launch (time it with events on `stream`)."""
+    import torch
+
+    if not (isinstance(feats, torch.Tensor) and feats.is_cuda and feats.dtype == torch.float32):
+        raise TypeError("feats must be a float32 CUDA tensor")
+    if not feats.is_contiguous() or feats.dim() != 2:
+        raise ValueError("feats must be a contiguous [n][F] tensor")
+    n = feats.shape[0]
+    if out_sums is None:
+        out_sums = torch.empty(n, dtype=torch.float32, device=feats.device)
+    visits = C.c_int64()
+    _check(lib().mlt_walk_peak(_stream_ptr(stream), int(model_id), _dptr(feats), n, int(rounds), _dptr(out_sums),
+                               C.byref(visits)))
+    return out_sums, int(visits.value)
 
 
 def last_survivor_count(stream=None) -> int:

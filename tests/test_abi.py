@@ -169,3 +169,16 @@ def test_half_table_loader_rejects(case):
 def test_wait_selftest_rejects_limits(L, limit):
     # rejected on the host, before any CUDA call
     assert L.mlt_selftest_wait_timeout(None, limit) == -1
+
+
+def test_walk_peak_rejects_bad_arguments(L):
+    # rejected on the host, before any CUDA call
+    mlt.set_num_features(4)
+    buf = C.c_void_p(16)
+    out = C.c_int64()
+    assert L.mlt_walk_peak(None, 2, buf, 10, 1, buf, C.byref(out)) == -1  # model A
+    assert L.mlt_walk_peak(None, 0, buf, 0, 1, buf, C.byref(out)) == -1  # n
+    assert L.mlt_walk_peak(None, 0, buf, 10, 0, buf, C.byref(out)) == -1  # rounds
+    assert L.mlt_walk_peak(None, 0, None, 10, 1, buf, C.byref(out)) == -1
+    assert L.mlt_walk_peak(None, 0, buf, 10, 1, buf, None) == -1
+    assert L.mlt_walk_peak(None, 0, buf, 10, 1, buf, C.byref(out)) == -2  # nothing loaded
