@@ -638,6 +638,7 @@ def run_ours(args):
             "bound": "hbm", "achieved": step_bytes / (ms_per_step / 1e3) / 1e9, "peak": hbm_gbs,
             "unit": "GB/s", "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / hbm_gbs,
             "peak_source": peak_src, "bytes_per_step": step_bytes,
+            "frac_of_nominal_7900": step_bytes / (ms_per_step / 1e3) / 1e9 / 7900.0,
             "dominant_kernel_gbs": dom_bytes / (dom_ms / 1e3) / 1e9,
         },
         "e2e": {"value": world * n / e2e_s, "unit": "candidates/s",
