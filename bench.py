@@ -32,7 +32,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "candidates screened/sec (V filter + P score + top-k) at 1 GB300; % HBM roofline"
-DEFAULT_CONFIG = 2
+DEFAULT_WORKLOAD = 2
 L2_FLUSH_BYTES = 256 << 20
 SM_COUNT = 152
 SM_MAX_MHZ_NOMINAL = 2070.0
@@ -144,7 +144,7 @@ def run_reference(args):
         return 0
     from paper_2411_10764_gb300 import workloads as W
 
-    w = W.make_workload(args.config, seed=args.seed, n=args.n)
+    w = W.make_workload(args.workload, seed=args.seed, n=args.n)
     import oracle as O
 
     O.build()
@@ -182,7 +182,7 @@ def run_reference(args):
 
 def config_dict(w):
     c = w.cfg
-    return {"workload": f"{c.name} (config {c.id})", "n": w.n, "F": c.F,
+    return {"workload": f"{c.name} (workload {c.id})", "n": w.n, "F": c.F,
             "v_trees": c.v_trees, "v_depth": c.v_depth, "p_trees": c.p_trees, "p_depth": c.p_depth,
             "thr": c.thr, "k": c.k, "seed": None,
             "l2": "flushed before every timed step (256 MB device write, outside the step events)"}
@@ -208,7 +208,7 @@ def walk_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def dram_traffic(config: int, phase: str):
+def dram_traffic(workload: int, phase: str):
     """DRAM bytes per launch of the phase's walk kernel from the committed
     ncu capture, or None if there is none or the walk sources changed since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
@@ -219,7 +219,7 @@ def dram_traffic(config: int, phase: str):
         return None
     if tr.get("walk_source_hash") != walk_source_hash():
         return None
-    ent = tr.get(f"config{config}:{phase}")
+    ent = tr.get(f"workload{workload}:{phase}")
     return ent.get("dram_bytes_per_launch") if ent else None
 
 
@@ -293,7 +293,7 @@ def run_ours(args):
     from paper_2411_10764_gb300 import workloads as W
 
     seed = args.seed + rank
-    w = W.make_workload(args.config, seed=seed, n=args.n)
+    w = W.make_workload(args.workload, seed=seed, n=args.n)
     mlt.load_workload_models(w)
     n, k, thr = w.n, w.k, w.thr
     pv = torch.empty(n, dtype=torch.float32, device=dev)
@@ -616,7 +616,7 @@ def run_ours(args):
     dom_bytes = (cnt["feat_bytes"] + cnt["v_table_bytes"]) if dominant == "v_pass" else \
         (cnt["survivor_feat_bytes"] + cnt["p_table_bytes"])
     step_bytes = cnt["feat_bytes"] + cnt["v_table_bytes"] + cnt["p_table_bytes"]
-    traffic = dram_traffic(args.config, dominant)
+    traffic = dram_traffic(args.workload, dominant)
     line = {
         "metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -671,7 +671,8 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=DEFAULT_CONFIG)
+    ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD,
+                    help="workload 1-5 (1 tiny, 2 gemm, 3 sa-batch, 4 conv2d decoded, 5 skewed-nan)")
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")

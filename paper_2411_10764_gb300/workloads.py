@@ -157,7 +157,7 @@ def _feature_chunk(cfg: ScreenConfig, seed: int, chunk: int, rows: int) -> np.nd
             src = rng.integers(0, rows, size=n_dup)
             x[dst] = x[src]
     else:
-        raise ValueError(f"config {cfg.id} has no stored feature matrix")
+        raise ValueError(f"workload {cfg.id} has no stored feature matrix")
     assert x.shape == (rows, cfg.F)
     return np.ascontiguousarray(x, dtype=np.float32)
 

@@ -186,7 +186,7 @@ def test_decoded_screen_equals_materialised_screen():
     torch.cuda.synchronize()
 
 
-def test_full_size_config2_all_outputs():
+def test_full_size_workload2_all_outputs():
     w = W.make_workload(2, seed=1)
     assert_parity(gpu_screen(w), oracle_screen(w))
 
@@ -215,7 +215,7 @@ def _sampled_full_size(cid, n_sample=1500):
     assert_same_bits(gpf[rows], opf, "perf (sampled)")
     assert_pvalid(gpv[rows], opv)
     n_near = int(np.sum(np.abs(gpf[finite] - kth) <= 1e-6 * abs(kth)))
-    print(f"config {cid}: survivors {gs}/{w.n}, {rows.size} rows checked, "
+    print(f"workload {cid}: survivors {gs}/{w.n}, {rows.size} rows checked, "
           f"{n_near} scores within 1e-6 of the k-th")
 
 

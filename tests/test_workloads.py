@@ -45,7 +45,7 @@ def test_feature_rows_are_a_prefix_across_sizes():
     assert np.array_equal(small, large[:1000])
 
 
-def test_config5_missing_values_duplicates_and_tree_size():
+def test_workload5_missing_values_duplicates_and_tree_size():
     w = W.make_workload(5, seed=1, n=65536)
     assert 0.28 < np.isnan(w.feats).mean() < 0.32
     _, counts = np.unique(w.feats.view(np.uint32).reshape(65536, -1), axis=0, return_counts=True)
@@ -55,7 +55,7 @@ def test_config5_missing_values_duplicates_and_tree_size():
     assert 2600 < per_tree < 3200  # about 2,890 nodes per tree
 
 
-def test_config2_knob_features_and_zeros():
+def test_workload2_knob_features_and_zeros():
     x = W.make_features(W.CONFIGS[2], 1, 20000)
     knobs = x[:, :12]
     assert set(np.unique(knobs).tolist()) == set(float(i) for i in range(11))
