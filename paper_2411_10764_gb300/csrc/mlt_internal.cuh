@@ -139,12 +139,10 @@ struct DecodeParams {
 // ---------------------------------------------------------------------------
 // The P pass histograms the top kTopBits bits of every rank key; the top-k
 // kernel reads it to find the bucket holding the k-th key, collects the keys
-// of that bucket and above (normally a few thousand), and sorts them in one
-// CTA.  kCollectCap is the most keys that sort in shared memory; a larger
-// collection (heavy ties) is narrowed by a radix select first.
+// of that bucket and above (a few hundred to a few thousand here), and one
+// CTA narrows them to exactly k by radix digits and orders those.
 constexpr int kTopBits = 12;
 constexpr int kTopBins = 1 << kTopBits;
-constexpr int kCollectCap = 16384;
 
 struct SelectState {
   unsigned int survivors;  // valid candidates of the current batch
