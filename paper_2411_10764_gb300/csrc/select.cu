@@ -12,11 +12,12 @@
 // counts the keys' top 12 bits in a histogram.  One top-k kernel then finds
 // the histogram bucket holding the k-th key, collects every key in that
 // bucket or above (a few hundred to a few thousand for the workloads here),
-// and the last CTA to finish (ticket counter, no waiting) narrows them to
-// exactly the k best with an exact most-significant-digit radix select
-// (8-bit digits below the bucket's bits, counted in shared memory) and
-// orders those: by counting for each key the larger ones (up to 512 keys),
-// else by a bitonic sort.
+// and the last CTA to finish (ticket counter, no waiting) orders them.  Up to
+// 512 collected keys are ranked directly (each key counts the larger ones);
+// a larger collection is first narrowed to exactly the k best with an exact
+// most-significant-digit radix select (8-bit digits below the bucket's bits,
+// counted in shared memory), whose keys are then ranked the same way (k <=
+// 512) or sorted (bitonic).
 #include "mlt_internal.cuh"
 
 namespace mlt {
@@ -24,7 +25,8 @@ namespace {
 
 constexpr int kTopkThreads = 512;
 constexpr int kSortMin = 8192;  // collected keys held in shared memory
-constexpr unsigned kRankMax = 512;  // order by rank counting up to this many keys
+constexpr unsigned kRankMax = 512;    // order by rank counting up to this many keys
+constexpr unsigned kDirectMax = 512;  // rank a collection this small without narrowing it
 
 __global__ void __launch_bounds__(256)
     k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n, const StreamState* ss) {
@@ -63,21 +65,50 @@ __device__ void sort_desc(unsigned long long* sk, int n2) {
   }
 }
 
-// Rank of every key among out_keys[0, kk) (keys unique), by counting the
-// larger ones: no barrier, cheaper than a bitonic sort for a few hundred
-// keys.  out_keys[kk] must be readable (0 when kk is odd: smaller than any key).
-__device__ void write_by_rank(const unsigned long long* out_keys, unsigned kk, long long base, int64_t* out) {
-  const ulonglong2* pairs = reinterpret_cast<const ulonglong2*>(out_keys);
-  const unsigned n_pairs = (kk + 1u) >> 1;
-  for (unsigned i = threadIdx.x; i < kk; i += blockDim.x) {
-    const unsigned long long key = out_keys[i];
-    unsigned r = 0;
-    for (unsigned j = 0; j < n_pairs; ++j) {
-      const ulonglong2 q = pairs[j];
-      r += (q.x > key) + (q.y > key);
+// Rank of every key among ks[0, m) (keys unique), by counting the larger
+// ones; the key of rank r < kk goes to out[r].  p threads share a key (a
+// power of two up to 32, as many as the block holds) and add their partial
+// counts with shuffles: no barrier, cheaper than a bitonic sort for a few
+// hundred keys.  ks[m] must be readable (0 when m is odd: below any key).
+__device__ void rank_and_write(const unsigned long long* ks, unsigned m, unsigned kk, long long base,
+                               int64_t* out) {
+  const ulonglong2* pairs = reinterpret_cast<const ulonglong2*>(ks);
+  const unsigned n_pairs = (m + 1u) >> 1;
+  unsigned p = 1;
+  while (p < 32u && 2u * p * m <= blockDim.x) p <<= 1;
+  if (p == 1) {  // one thread per key: a plain loop the compiler unrolls
+    for (unsigned i = threadIdx.x; i < m; i += blockDim.x) {
+      const unsigned long long key = ks[i];
+      unsigned r = 0;
+      for (unsigned j = 0; j < n_pairs; ++j) {
+        const ulonglong2 q = pairs[j];
+        r += (q.x > key) + (q.y > key);
+      }
+      if (r < kk) {
+        const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull);
+        out[r] = base + static_cast<long long>(pos);
+      }
     }
-    const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull);
-    out[r] = base + static_cast<long long>(pos);
+    return;
+  }
+  const unsigned span = m * p;
+  for (unsigned t0 = 0; t0 < span; t0 += blockDim.x) {  // the same trip count in every thread
+    const unsigned t = t0 + threadIdx.x;
+    const unsigned i = t / p, part = t % p;
+    unsigned long long key = 0;
+    unsigned r = 0;
+    if (t < span) {
+      key = ks[i];
+      for (unsigned j = part; j < n_pairs; j += p) {
+        const ulonglong2 q = pairs[j];
+        r += (q.x > key) + (q.y > key);
+      }
+    }
+    for (unsigned o = 1; o < p; o <<= 1) r += __shfl_xor_sync(0xFFFFFFFFu, r, o);
+    if (t < span && part == 0 && r < kk) {
+      const uint32_t pos = 0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull);
+      out[r] = base + static_cast<long long>(pos);
+    }
   }
 }
 
@@ -164,6 +195,15 @@ __global__ void __launch_bounds__(kTopkThreads)
     const bool in_smem = m <= static_cast<unsigned>(kSortMin);
     if (in_smem)
       for (unsigned i = tid; i < m; i += T) sk[i] = __ldcg(cand + i);
+    if (m < kk && tid == 0) atomicOr(err, kErrSelect);  // the histogram promised kk
+    if (m <= kDirectMax) {
+      // a small collection: rank every collected key directly
+      if (tid == 0 && (m & 1u)) sk[m] = 0ull;
+      __syncthreads();
+      rank_and_write(sk, m, kk, base, out);
+      for (int r = static_cast<int>(kk) + tid; r < k; r += T) out[r] = -1;
+      return;
+    }
     auto key_at = [&](unsigned i) { return in_smem ? sk[i] : __ldcg(cand + i); };
     unsigned long long mask = ~0ull << (64 - kTopBits);
     unsigned long long prefix = bin << (64 - kTopBits);
@@ -224,7 +264,7 @@ __global__ void __launch_bounds__(kTopkThreads)
     if (tid == 0 && (kk & 1u)) out_keys[kk] = 0ull;  // pad for the pairwise rank loop (kk odd < n2k)
     __syncthreads();
     if (kk <= kRankMax) {
-      write_by_rank(out_keys, kk, base, out);
+      rank_and_write(out_keys, kk, kk, base, out);
     } else {
       int n2 = 1;
       while (n2 < static_cast<int>(kk)) n2 <<= 1;
