@@ -52,10 +52,16 @@ def oracle_screen(w, thr=None, k=None, feats=None):
     return pv, pf, tk, s
 
 
-def assert_same_bits(a, b, what):
-    a = np.asarray(a, np.float32)
-    b = np.asarray(b, np.float32)
-    bad = np.nonzero(a.view(np.uint32) != b.view(np.uint32))[0]
+def assert_same_bits(a, b, what, nan_equal=False):
+    """Bit-for-bit equality of float32 arrays.  With nan_equal, a NaN matches
+    any NaN: IEEE 754 leaves the bits of a NaN an operation generates to the
+    implementation (the GPU gives 0x7FFFFFFF, an Arm host 0x7FC00000)."""
+    a = np.asarray(a, np.float32).ravel()
+    b = np.asarray(b, np.float32).ravel()
+    diff = a.view(np.uint32) != b.view(np.uint32)
+    if nan_equal:
+        diff &= ~(np.isnan(a) & np.isnan(b))
+    bad = np.nonzero(diff)[0]
     assert bad.size == 0, f"{what}: {bad.size} mismatches, first at {bad[:5]}: {a[bad[:5]]} vs {b[bad[:5]]}"
 
 

@@ -1,0 +1,86 @@
+"""GPU parity of the on-device knob decoder on random knob spaces and random
+feature programs: every opcode; operands that are constants, knob values or
+earlier features; option values and constants of both signs, zero,
+subnormal and huge magnitudes (so divisions by zero, overflow to infinity and
+NaN arise).  Decoded knobs and features are compared with the oracle bit for
+bit (a generated NaN matches any NaN: IEEE 754 leaves its bits to the
+implementation), and screening straight from candidate indices is compared
+with the oracle's screening of its own decoded rows."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2411_10764_gb300 import mlt
+from paper_2411_10764_gb300 import workloads as W
+from screening import THREADS, assert_parity, assert_same_bits, gpu_screen, oracle_screen
+
+pytestmark = pytest.mark.gpu
+
+CASES = 20
+SPECIAL = np.array([0.0, -0.0, 1.0, -1.0, 2.0, 0.5, 3.0, 7.0, 1e-40, -1e-40, 1e30, -1e30, 0.1, 1024.0],
+                   np.float32)
+
+
+def _values(rng, size):
+    v = np.where(rng.random(size) < 0.5, SPECIAL[rng.integers(0, SPECIAL.size, size)],
+                 (rng.standard_normal(size) * 10.0 ** rng.integers(-3, 4, size)).astype(np.float32))
+    return v.astype(np.float32)
+
+
+def _decoder(case):
+    rng = np.random.default_rng(9100 + case)
+    n_knobs = int(rng.integers(1, 17))
+    radices = rng.integers(1, 13, size=n_knobs).astype(np.int32)
+    option_values = _values(rng, int(radices.sum()))
+    F = int(rng.integers(1, 61))
+    prog = np.zeros(F, dtype=W.OP_DTYPE)
+    for f in range(F):
+        prog[f]["op"] = int(rng.integers(0, 12))
+        for field in ("a", "b"):
+            kind = rng.integers(0, 3)
+            if kind == 0 or (kind == 2 and f == 0):
+                prog[f][field] = -1
+            elif kind == 1:
+                prog[f][field] = int(rng.integers(0, n_knobs))
+            else:
+                prog[f][field] = n_knobs + int(rng.integers(0, f))
+        prog[f]["c"] = _values(rng, 1)[0]
+    return W.Decoder(radices, option_values, prog, []), rng
+
+
+@pytest.mark.parametrize("case", range(CASES))
+def test_random_programs_decode_bit_exact(case):
+    d, rng = _decoder(case)
+    space = d.space
+    n = int(min(space, rng.integers(1, 5001)))
+    first = int(rng.integers(0, space - n + 1))
+    knobs, feats = mlt.decode_knobs(d.radices, d.option_values, d.program, first, n)
+    mlt.sync_status()
+    ok, of = O.features(d.radices, d.option_values, d.program, first, n, threads=THREADS)
+    assert np.array_equal(knobs.cpu().numpy(), ok)
+    # every number bit for bit; a NaN the program generates matches any NaN
+    assert_same_bits(feats.cpu().numpy(), of, "decoded features", nan_equal=True)
+    assert np.array_equal(np.isnan(feats.cpu().numpy()), np.isnan(of))
+
+
+@pytest.mark.parametrize("case", range(CASES))
+def test_random_programs_screen_from_indices(case):
+    d, rng = _decoder(case)
+    space = d.space
+    n = int(min(space, rng.integers(1, 20001)))
+    first = int(rng.integers(0, space - n + 1))
+    F = d.program.size
+    _, sample = O.features(d.radices, d.option_values, d.program, first, min(n, 2048), threads=THREADS)
+    sample = np.where(np.isfinite(sample), sample, np.nan).astype(np.float32)
+    th = W._QuantileThresholds(sample)
+    thr = float(rng.choice([0.2, 0.5, 0.8]))
+    k = int(rng.choice([1, 16, 300]))
+    cfg = W.ScreenConfig(950 + case, f"decode-fuzz-{case}", n, F, 1, 1, 1, 1, thr, k, None, decoded=True)
+    shapes = [(str(rng.choice(["full", "unbalanced"])), int(rng.integers(1, 40))) for _ in range(2)]
+    ens = []
+    for (shape, n_trees), which in zip(shapes, ("V", "P")):
+        depth = int(rng.integers(1, 9)) if shape == "full" else int(rng.integers(2, 13))
+        ens.append(W.make_ensemble(cfg, which, th, 61 + case, n_trees=n_trees, depth=depth, split_prob=0.8,
+                                   shape=shape))
+    w = W.Workload(cfg, n, None, d, first, ens[0], ens[1], thr, k)
+    assert_parity(gpu_screen(w), oracle_screen(w))
