@@ -84,3 +84,33 @@ def test_random_programs_screen_from_indices(case):
                                    shape=shape))
     w = W.Workload(cfg, n, None, d, first, ens[0], ens[1], thr, k)
     assert_parity(gpu_screen(w), oracle_screen(w))
+
+
+@pytest.mark.parametrize("case", range(6))
+def test_indices_past_32_bits_decode_bit_exact(case):
+    """Knob spaces of 2^35 .. 2^56 candidates (10 to 14 knobs of 12 to 16
+    options): batches that straddle index 2^32, where the decoder switches
+    from 32-bit to 64-bit digit division, batches at the end of the space and
+    one in between."""
+    d, rng = _decoder(100 + case)
+    n_knobs = int(rng.integers(10, 15))
+    radices = rng.integers(12, 17, size=n_knobs).astype(np.int32)
+    option_values = _values(rng, int(radices.sum()))
+    prog = d.program.copy()
+    for f in range(prog.size):  # operands name this space's knobs
+        for field in ("a", "b"):
+            v = int(prog[f][field])
+            if v >= d.n_knobs:
+                prog[f][field] = n_knobs + (v - d.n_knobs)
+            elif v >= 0:
+                prog[f][field] = v % n_knobs
+    d = W.Decoder(radices, option_values, prog, [])
+    space = d.space
+    assert space > 2 ** 34
+    n = 3000
+    for first in (2 ** 32 - n // 2, space - n, int(rng.integers(2 ** 33, space - n))):
+        knobs, feats = mlt.decode_knobs(d.radices, d.option_values, d.program, first, n)
+        mlt.sync_status()
+        ok, of = O.features(d.radices, d.option_values, d.program, first, n, threads=THREADS)
+        assert np.array_equal(knobs.cpu().numpy(), ok)
+        assert_same_bits(feats.cpu().numpy(), of, "decoded features", nan_equal=True)
