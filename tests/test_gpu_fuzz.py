@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 from paper_2411_10764_gb300 import workloads as W
-from screening import assert_parity, gpu_screen, oracle_screen
+from screening import assert_parity, assert_same_bits, gpu_screen, oracle_screen
 
 pytestmark = pytest.mark.gpu
 
@@ -95,3 +95,32 @@ def test_random_problem_half_tables_match_rounded_oracle(case):
     opv, opf, valid, _ = O.screen_rows(x, O.half_ensemble(w.v), O.half_ensemble(w.p), w.thr, threads=THREADS)
     otk, s = O.topk(opf, valid, w.k)
     assert_parity(got, (opv, opf, otk, s))
+
+
+@pytest.mark.parametrize("case", range(CASES // 2))
+def test_random_rerank_matches_oracle(case):
+    """Model A (complete or unbalanced, depth 1 to 14, 1 to 400 trees) reranks
+    a random candidate list (padding, duplicates, up to 3,000 entries) of the
+    same random problems; scores bit for bit and the final order exactly."""
+    import torch
+
+    import oracle as O
+    from paper_2411_10764_gb300 import mlt
+
+    w = _draw_case(case)
+    rng = np.random.default_rng(8000 + case)
+    shape = str(rng.choice(["full", "unbalanced"]))
+    depth = int(rng.integers(1, 11)) if shape == "full" else int(rng.integers(2, 15))
+    th = W._QuantileThresholds(np.where(np.isfinite(w.feats), w.feats, np.nan)[:4096])
+    a = W.make_ensemble(w.cfg, "A", th, 77 + case, n_trees=int(rng.integers(1, 401)), depth=depth,
+                        split_prob=float(rng.uniform(0.5, 0.95)), shape=shape)
+    m = int(rng.integers(1, 3001))
+    cand = rng.integers(-1, w.n, size=m).astype(np.int64)  # -1: padding; duplicates likely
+    n_final = int(rng.integers(1, m + 5))
+    mlt.load_workload_models(w)
+    mlt.load_ensemble(mlt.MLT_MODEL_A, a.nodes, a.n_trees, a.depth)
+    sc, fin = mlt.rerank(torch.from_numpy(w.feats).cuda(), torch.from_numpy(cand).cuda(), n_final)
+    mlt.sync_status()
+    osc, ofin = O.rerank(w.feats, cand, a, n_final)
+    assert_same_bits(sc.cpu().numpy(), osc, "A scores")
+    assert np.array_equal(fin.cpu().numpy(), ofin)
