@@ -124,3 +124,42 @@ def test_random_rerank_matches_oracle(case):
     osc, ofin = O.rerank(w.feats, cand, a, n_final)
     assert_same_bits(sc.cpu().numpy(), osc, "A scores")
     assert np.array_equal(fin.cpu().numpy(), ofin)
+
+
+def _expected_prefix(valid, n, batch, target):
+    """(consumed, kept, batches) of the accumulation rule on oracle decisions."""
+    kept = 0
+    for b, b0 in enumerate(range(0, n, batch)):
+        b1 = min(n, b0 + batch)
+        kept += int(valid[b0:b1].sum())
+        if kept >= target:
+            return b1, kept, b + 1
+    return n, kept, -(-n // batch)
+
+
+@pytest.mark.parametrize("case", range(CASES // 2))
+def test_random_accumulation_matches_oracle(case):
+    """Batched accumulation (mlt_screen_until) over the random problems with
+    random batch sizes and targets: the consumed prefix, the kept count and
+    the batch count follow the accumulation rule on the oracle's decisions;
+    the top-k and the prefix's scores match the oracle."""
+    import torch
+
+    import oracle as O
+    from paper_2411_10764_gb300 import mlt
+    from screening import THREADS, assert_pvalid
+
+    w = _draw_case(case)
+    rng = np.random.default_rng(8500 + case)
+    batch = int(rng.integers(32, max(33, w.n + 100)))
+    target = int(rng.integers(1, max(2, w.n)))
+    mlt.load_workload_models(w)
+    pv, pf, tk, stats = mlt.screen_until(torch.from_numpy(w.feats).cuda(), batch, target, w.thr, w.k)
+    mlt.sync_status()
+    opv, opf, valid, _ = O.screen_rows(w.feats, w.v, w.p, w.thr, threads=THREADS)
+    consumed, kept, batches = _expected_prefix(valid, w.n, batch, target)
+    assert stats.cpu().tolist() == [consumed, kept, batches]
+    want, _ = O.topk(opf[:consumed], valid[:consumed], w.k)
+    assert np.array_equal(tk.cpu().numpy(), want)
+    assert_same_bits(pf.cpu().numpy()[:consumed], opf[:consumed], "perf (consumed prefix)")
+    assert_pvalid(pv.cpu().numpy()[:consumed], opv[:consumed])
