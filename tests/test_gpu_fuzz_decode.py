@@ -114,3 +114,52 @@ def test_indices_past_32_bits_decode_bit_exact(case):
         ok, of = O.features(d.radices, d.option_values, d.program, first, n, threads=THREADS)
         assert np.array_equal(knobs.cpu().numpy(), ok)
         assert_same_bits(feats.cpu().numpy(), of, "decoded features", nan_equal=True)
+
+
+def _gpu_sa(d, parent, ps, kd, dd, lu, temperature, thr):
+    import torch
+
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a).astype(dt)).cuda()
+    nxt, nsc, acc = mlt.sa_step(d.radices, d.option_values, d.program, t(parent, np.int64), t(ps, np.float32),
+                                t(np.asarray(kd, np.uint32).view(np.int32), np.int32),
+                                t(np.asarray(dd, np.uint32).view(np.int32), np.int32), t(lu, np.float32),
+                                temperature, thr)
+    mlt.sync_status()
+    return nxt.cpu().numpy(), nsc.cpu().numpy(), acc.cpu().numpy()
+
+
+@pytest.mark.parametrize("case", range(10))
+def test_random_explorer_steps_match_oracle(case):
+    """Three proposal steps of random chains over the random knob spaces and
+    programs (random V and P ensembles on the decoded features, inactive
+    chains, temperatures from hot to cold): next indices, chain scores and
+    acceptances equal the oracle's."""
+    d, rng = _decoder(case)
+    space = d.space
+    F = d.program.size
+    _, sample = O.features(d.radices, d.option_values, d.program, 0, int(min(space, 2048)), threads=THREADS)
+    sample = np.where(np.isfinite(sample), sample, np.nan).astype(np.float32)
+    th = W._QuantileThresholds(sample)
+    thr = float(rng.choice([0.3, 0.5, 0.7]))
+    cfg = W.ScreenConfig(970 + case, f"sa-fuzz-{case}", 1, F, 1, 1, 1, 1, thr, 1, None, decoded=True)
+    v = W.make_ensemble(cfg, "V", th, 81 + case, n_trees=int(rng.integers(1, 60)), depth=int(rng.integers(1, 9)),
+                        shape="full")
+    p = W.make_ensemble(cfg, "P", th, 82 + case, n_trees=int(rng.integers(1, 60)), depth=int(rng.integers(2, 13)),
+                        split_prob=0.8, shape="unbalanced")
+    mlt.set_num_features(F)
+    mlt.load_ensemble(mlt.MLT_MODEL_V, v.nodes, v.n_trees, v.depth)
+    mlt.load_ensemble(mlt.MLT_MODEL_P, p.nodes, p.n_trees, p.depth)
+    m = int(rng.integers(1, 5000))
+    parent = rng.integers(0, space, size=m).astype(np.int64)
+    parent[rng.random(m) < 0.05] = -1  # inactive chains
+    ps = np.full(m, -np.inf, np.float32)
+    for step, temperature in enumerate([4.0, 1.0, 0.1]):
+        kd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+        dd = rng.integers(0, 2 ** 32, size=m, dtype=np.uint64).astype(np.uint32)
+        lu = np.log(rng.random(m)).astype(np.float32)
+        g = _gpu_sa(d, parent, ps, kd, dd, lu, temperature, thr)
+        o = O.sa_step(d.radices, d.option_values, d.program, v, p, parent, ps, kd, dd, lu, temperature, thr)
+        assert np.array_equal(g[0], o[0]), step
+        assert_same_bits(g[1], o[1], f"chain scores step {step}")
+        assert np.array_equal(g[2], o[2]), step
+        parent, ps = o[0], o[1]
