@@ -171,9 +171,13 @@ int mlt_screen(void *stream, const float *feats, int64_t n, float thr, int k,
  *   - every call shares the one array: calls whose GPU work overlaps (for
  *     example on two streams without ordering) race and give undefined
  *     results;
+ *   - each call clears the array's selection state before its kernels
+ *     run, so a call that stopped part-way leaves nothing behind for the
+ *     next one;
  *   - a device-side error bit (a bounded wait that gave up) lives in the
- *     array too; it is cleared by the next call, and mlt_sync_status does
- *     not report it.
+ *     array too; mlt_sync_status on the same device reports it (as for the
+ *     other entry points) and clears it.  A call that met such an error
+ *     leaves its outputs undefined.
  * Models V and P must have been loaded with mlt_load_ensemble beforehand. */
 int mlt_screen_noalloc(void *stream, const float *feats, int64_t n, float thr, int k,
                        float *out_pvalid, float *out_perf, int64_t *out_topk);
@@ -312,6 +316,25 @@ int mlt_sync_status(void *stream);
  * MLT_ETIMEOUT and the device stays usable.  No fault, trap or endless
  * loop is involved.  Asynchronous. */
 int mlt_selftest_wait_timeout(void *stream, int64_t limit_ns);
+
+/* Failure-detection self-test inside the screening path: arms a one-shot
+ * so that the next screening call whose model V has a full table (depth
+ * <= 10) makes V-pass CTA `cta` (clamped to the last CTA) wait for its
+ * first tree chunk on a barrier phase that nothing completes.  That wait
+ * gives up after limit_ns (1e6 .. 2e9 ns); the CTA lets its copies land,
+ * records the timeout, and still completes its tile's bookkeeping (none of
+ * its candidates valid), so the call's other results stay consistent and
+ * the next call is unaffected.  mlt_sync_status then reports MLT_ETIMEOUT.
+ * No fault, trap or endless loop is involved.  Host-only bookkeeping. */
+int mlt_selftest_walk_timeout(int cta, int64_t limit_ns);
+
+/* Test support: writes `value` into the four counters (survivor count,
+ * collected keys, two CTA tickets) of the selection state that the
+ * allocating entry points (static_scratch = 0) or mlt_screen_noalloc
+ * (static_scratch != 0) use on the current device, as a call that stopped
+ * part-way could leave them.  Every screening call clears that state before
+ * its kernels run, so results must not change.  Synchronous. */
+int mlt_selftest_poison_state(int static_scratch, uint32_t value);
 
 /* Number of valid candidates found by the last screening call (waits for
  * `stream`). */

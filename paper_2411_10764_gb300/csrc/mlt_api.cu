@@ -128,6 +128,11 @@ ScratchOwner g_scr;
 int g_optin = -1;
 int g_sms = -1;
 ShapeOverride g_shape[3];
+// failure-detection self-test, armed by mlt_selftest_walk_timeout: the next
+// full-table V pass makes CTA g_stall_cta wait on a barrier phase that
+// nothing completes, for g_stall_ns (one shot)
+int g_stall_cta = -1;
+unsigned long long g_stall_ns = 0;
 
 size_t align16(size_t v) { return (v + 15) & ~static_cast<size_t>(15); }
 
@@ -484,6 +489,10 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   av.chunk_trees = sv.chunk_trees;
   av.nbuf = sv.nbuf;
   av.max_depth = V.depth;
+  // every call starts from a fresh selection state: its tickets decide which
+  // CTA scans the tile counts and ranks the keys, so a count left behind by
+  // an earlier call (one that stopped part-way) must not carry over
+  MLT_CUDA(cudaMemsetAsync(s.state, 0, sizeof(SelectState), st), "reset selection state");
   cudaEvent_t* ev = nullptr;
   if (g_profile && profile_ok) {
     if (g_events_used + kPhases + 1 > g_events.size()) {
@@ -498,6 +507,11 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
     MLT_CUDA(cudaEventRecord(ev[0], st), "cudaEventRecord");
   }
   const long long tiles_v = (n + sv.threads - 1) / sv.threads;
+  if (g_stall_cta >= 0 && V.kind != kTableCompact && tiles_v > 0) {
+    av.stall_cta = static_cast<int>(std::min<long long>(g_stall_cta, tiles_v - 1));
+    av.stall_ns = g_stall_ns;
+    g_stall_cta = -1;
+  }
   MLT_CUDA(dec ? launch_traverse_dec(V, av, *dec, sv, tiles_v, st) : launch_traverse(V, av, sv, tiles_v, st),
            "V pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[1], st), "cudaEventRecord");
@@ -532,6 +546,10 @@ int noalloc_scratch(int dev, Scratch* out) {
   if (g_noalloc_base[dev] == nullptr) {
     void* p = nullptr;
     MLT_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch), "cudaGetSymbolAddress(static scratch)");
+    // the error word starts at zero (it is cleared again whenever
+    // mlt_sync_status reads it)
+    MLT_CUDA(cudaMemset(static_cast<unsigned char*>(p) + kErr, 0, sizeof(unsigned int)),
+             "clear static error word");
     g_noalloc_base[dev] = static_cast<unsigned char*>(p);
   }
   unsigned char* b = g_noalloc_base[dev];
@@ -836,9 +854,9 @@ int mlt_screen_noalloc(void* stream, const float* feats, int64_t n, float thr, i
   rc = noalloc_scratch(dev, &s);
   if (rc != MLT_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  // the array keeps the previous call's contents: the error word must start
-  // at zero (every other piece is rewritten before it is read)
-  MLT_CUDA(cudaMemsetAsync(s.err, 0, sizeof(unsigned int), st), "clear static error word");
+  // the array keeps the previous call's contents; the selection state is
+  // cleared at the start of the sequence, the error word only when
+  // mlt_sync_status reads it (so a fault of this call stays visible)
   return run_screen_with(st, feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk, s, false);
 }
 
@@ -1126,11 +1144,23 @@ int mlt_decode_knobs(void* stream, const int32_t* radices, const float* option_v
 int mlt_sync_status(void* stream) {
   MLT_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream synchronize");
   std::lock_guard<std::mutex> lk(g_mu);
-  if (g_scr.err == nullptr) return MLT_OK;
+  // the allocating entry points' error word, and the static scratch's of
+  // mlt_screen_noalloc on the current device (read and cleared without any
+  // allocation)
+  unsigned int* words[2] = {g_scr.err, nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < mlt_noalloc::kMaxDevices &&
+      g_noalloc_base[dev] != nullptr)
+    words[1] = reinterpret_cast<unsigned int*>(g_noalloc_base[dev] + mlt_noalloc::kErr);
   unsigned int word = 0;
-  MLT_CUDA(cudaMemcpy(&word, g_scr.err, sizeof(word), cudaMemcpyDeviceToHost), "error word read");
+  for (unsigned int* w : words) {
+    if (w == nullptr) continue;
+    unsigned int v = 0;
+    MLT_CUDA(cudaMemcpy(&v, w, sizeof(v), cudaMemcpyDeviceToHost), "error word read");
+    if (v != 0) MLT_CUDA(cudaMemset(w, 0, sizeof(v)), "error word reset");
+    word |= v;
+  }
   if (word == 0) return MLT_OK;
-  MLT_CUDA(cudaMemset(g_scr.err, 0, sizeof(word)), "error word reset");
   if (word & kErrWaitTimeout) return fail(MLT_ETIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
   if (word & kErrBadIndex) return fail(MLT_EINVAL, "a rerank candidate index was outside [0, n) (error word 0x%x)", word);
   return fail(MLT_ECUDA, "device-side bookkeeping error (error word 0x%x)", word);
@@ -1146,6 +1176,34 @@ int mlt_selftest_wait_timeout(void* stream, int64_t limit_ns) {
                                 static_cast<cudaStream_t>(stream)),
            "self-test launch");
   g_launches += 1;
+  return MLT_OK;
+}
+
+int mlt_selftest_walk_timeout(int cta, int64_t limit_ns) {
+  if (cta < 0) return fail(MLT_EINVAL, "cta must be >= 0");
+  if (limit_ns < 1000000LL || limit_ns > static_cast<int64_t>(kWaitLimitNs))
+    return fail(MLT_EINVAL, "limit_ns must lie in [1e6, %llu]", kWaitLimitNs);
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_stall_cta = cta;
+  g_stall_ns = static_cast<unsigned long long>(limit_ns);
+  return MLT_OK;
+}
+
+int mlt_selftest_poison_state(int static_scratch, uint32_t value) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  Scratch s;
+  if (static_scratch) {
+    rc = noalloc_scratch(dev, &s);
+  } else {
+    rc = ensure_scratch(0);
+    s = g_scr.s;
+  }
+  if (rc != MLT_OK) return rc;
+  const unsigned int words[4] = {value, value, value, value};  // survivors, n_cand, ticket, v_ticket
+  MLT_CUDA(cudaMemcpy(s.state, words, sizeof(words), cudaMemcpyHostToDevice), "state write");
   return MLT_OK;
 }
 

@@ -209,6 +209,11 @@ struct TraverseArgs {
   StreamState* stream;
   long long pos_base;      // position of the batch's first candidate in the call
   int p_wave;              // full-table P pass: CTAs one wave holds (0: the grid)
+  // failure-detection self-test (full tables): CTA `stall_cta` waits for its
+  // first chunk on a barrier phase that nothing completes and gives up after
+  // stall_ns (-1: no CTA does)
+  int stall_cta = -1;
+  unsigned long long stall_ns = 0;
 };
 
 struct ScreenShape {

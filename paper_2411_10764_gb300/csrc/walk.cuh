@@ -711,8 +711,11 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   __shared__ unsigned released[4];
   __shared__ int last_issued[4];  // latest chunk copied into each buffer
 
+  // bars[3] is never completed (nbuf <= 3): the self-test's stalled wait
+  const bool stall = static_cast<int>(blockIdx.x) == a.stall_cta;
   if (tid == 0) {
     for (int b = 0; b < a.nbuf; ++b) mbar_init(smem_u32(&bars[b]), 1);
+    if (stall) mbar_init(smem_u32(&bars[3]), 1);
     for (int b = 0; b < 4; ++b) {
       released[b] = 0u;
       last_issued[b] = b < n_chunks ? b : -1;
@@ -753,13 +756,20 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   // parked leaves: buffer p holds leaf t of candidate c at la[p] + t * row_bytes
   const uint32_t la0 = smem_u32(smem + leaf_off) + static_cast<uint32_t>(c) * 4u;
   const uint32_t la_step = static_cast<uint32_t>(a.chunk_trees) * row_bytes;
+  // wait for chunk ch in buffer b (bounded); the self-test's stalled CTA
+  // waits for its first chunk on bars[3] instead
+  auto chunk_wait = [&](int ch, int b) -> bool {
+    if (stall && ch == 0) return mbar_wait_bounded_ns(smem_u32(&bars[3]), 0u, a.stall_ns);
+    return mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
+  };
+  bool failed = false;
   if constexpr (kSyncFree) {
     const int n_warps = static_cast<int>(blockDim.x >> 5);
     const int lane = tid & 31;
     bool timed_out = false;
     for (int ch = 0; ch < n_chunks; ++ch) {
       const int b = ch % a.nbuf;
-      const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
+      const bool ok = chunk_wait(ch, b);
       if (!__all_sync(0xFFFFFFFFu, ok)) {
         timed_out = true;
         break;
@@ -793,12 +803,12 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
             mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(last_issued[b] / a.nbuf) & 1u);
         atomicOr(a.err, kErrWaitTimeout);
       }
-      return;
+      failed = true;
     }
   } else
   for (int ch = 0; ch < n_chunks; ++ch) {
     const int b = ch % a.nbuf;
-    const bool ok = mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
+    const bool ok = chunk_wait(ch, b);
     if (!__syncthreads_and(ok)) {
       if (tid == 0) {
         // let every copy still in flight land before the CTA's shared memory
@@ -808,7 +818,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
         mbar_wait_bounded(smem_u32(&bars[b]), static_cast<uint32_t>(ch / a.nbuf) & 1u);
         atomicOr(a.err, kErrWaitTimeout);
       }
-      return;
+      failed = true;
+      break;
     }
     const uint32_t tb = tbuf_a + static_cast<uint32_t>(b) * chunk_bytes;
     const int nt = min(a.chunk_trees, a.n_trees - ch * a.chunk_trees);
@@ -828,11 +839,16 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     __syncthreads();
     if (tid == 0 && ch + a.nbuf < n_chunks) issue(ch + a.nbuf, b);
   }
-  if (Q > 1 && q == 0) {
+  if (Q > 1 && q == 0 && !failed) {
     const uint32_t lp = la0 + static_cast<uint32_t>((n_chunks - 1) & 1) * la_step;
     const int np = live ? a.n_trees - (n_chunks - 1) * a.chunk_trees : 0;
     for (int t = 0; t < np; ++t) acc += lds_f32(lp + static_cast<uint32_t>(t) * row_bytes);
   }
+  // a CTA whose wait gave up still completes its tile's bookkeeping (no
+  // candidate of it valid, -inf scores): the V pass's tile count and ticket,
+  // which decide when the tile offsets are scanned and the selection state
+  // reset, stay consistent for this call and the next
+  if (failed) acc = -INFINITY;
   pdl_trigger();
   finish_tile(a, rowidx, tile0, rows_here, count, acc, TC);
 }

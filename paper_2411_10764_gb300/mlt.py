@@ -60,6 +60,8 @@ def lib(build_if_missing: bool = True):
             "mlt_load_ensemble_f16": [i32, P, i32, i32],
             "mlt_screen_host_batches": [P, i64, P, i64, f32, i32, P, P, P],
             "mlt_selftest_wait_timeout": [P, i64],
+            "mlt_selftest_walk_timeout": [i32, i64],
+            "mlt_selftest_poison_state": [i32, C.c_uint32],
             "mlt_free_ensemble": [i32],
             "mlt_validity_cut": [f32, P],
             "mlt_screen": [P, P, i64, f32, i32, P, P, P],
@@ -343,6 +345,19 @@ def selftest_wait_timeout(limit_ns: int, stream=None) -> None:
     """Launch the failure-detection self-test (a device wait that runs out);
     the next sync_status raises MltError with MLT_ETIMEOUT."""
     _check(lib().mlt_selftest_wait_timeout(_stream_ptr(stream), int(limit_ns)))
+
+
+def selftest_walk_timeout(cta: int, limit_ns: int) -> None:
+    """Arm the in-path self-test: the next screening call's V pass (full
+    table) makes CTA `cta` give up waiting for its first tree chunk after
+    limit_ns; the next sync_status raises MltError with MLT_ETIMEOUT."""
+    _check(lib().mlt_selftest_walk_timeout(int(cta), int(limit_ns)))
+
+
+def selftest_poison_state(value: int, static_scratch: bool = False) -> None:
+    """Write `value` into the selection state's counters (as a call that
+    stopped part-way could leave them); the next call must not notice."""
+    _check(lib().mlt_selftest_poison_state(1 if static_scratch else 0, C.c_uint32(value)))
 
 
 def walk_peak(feats, rounds: int, model_id: int = MLT_MODEL_V, out_sums=None, stream=None):

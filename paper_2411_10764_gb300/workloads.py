@@ -16,8 +16,10 @@ survivor rates below bracket.
 """
 from __future__ import annotations
 
+import concurrent.futures
 import dataclasses
 import math
+import os
 import statistics
 
 import numpy as np
@@ -166,9 +168,21 @@ def make_features(cfg: ScreenConfig, seed: int, n: int) -> np.ndarray:
     """Row-major [n][F] float32 features; rows come in fixed 65,536-row chunks,
     so a smaller n gives a prefix of the larger matrix."""
     out = np.empty((n, cfg.F), dtype=np.float32)
-    for c, a in enumerate(range(0, n, CHUNK_ROWS)):
+
+    def fill(c):
+        a = c * CHUNK_ROWS
         b = min(n, a + CHUNK_ROWS)
         out[a:b] = _feature_chunk(cfg, seed, c, CHUNK_ROWS)[: b - a]
+
+    chunks = range((n + CHUNK_ROWS - 1) // CHUNK_ROWS)
+    if len(chunks) <= 1:
+        for c in chunks:
+            fill(c)
+    else:
+        # every chunk has its own generator (seeded by its index), so the
+        # matrix does not depend on how the chunks are spread over threads
+        with concurrent.futures.ThreadPoolExecutor(min(len(chunks), os.cpu_count() or 1)) as ex:
+            list(ex.map(fill, chunks))
     return out
 
 

@@ -7,7 +7,8 @@ import numpy as np
 import oracle as O
 from paper_2411_10764_gb300 import mlt
 
-THREADS = max(1, min(32, os.cpu_count() or 1))
+# the oracle's rows are independent: split them over every host core
+THREADS = max(1, os.cpu_count() or 1)
 
 
 def gpu_screen(w, thr=None, k=None, feats=None):
@@ -52,6 +53,46 @@ def oracle_screen(w, thr=None, k=None, feats=None):
     return pv, pf, tk, s
 
 
+def oracle_screen_chunked(w, thr=None, k=None, chunk=1 << 20):
+    """The oracle's screening of the whole workload, `chunk` rows at a time
+    (a decoded workload is decoded by the oracle chunk by chunk, so its
+    feature matrix is never held whole), every chunk split over all host
+    cores; then one full sort for the top-k.  Returns (pvalid, perf, top-k,
+    survivors, margin_v)."""
+    thr = w.thr if thr is None else thr
+    k = w.k if k is None else k
+    n = w.n
+    pv = np.empty(n, np.float32)
+    pf = np.empty(n, np.float32)
+    valid = np.empty(n, bool)
+    mv = np.empty(n, np.float32)
+    for a in range(0, n, chunk):
+        b = min(n, a + chunk)
+        if w.decoder is None:
+            x = w.feats[a:b]
+        else:
+            d = w.decoder
+            _, x = O.features(d.radices, d.option_values, d.program, w.first_index + a, b - a,
+                              threads=THREADS)
+        pv[a:b], pf[a:b], valid[a:b], mv[a:b] = O.screen_rows(x, w.v, w.p, thr, threads=THREADS)
+    tk, s = O.topk(pf, valid, k, index_base=w.first_index)
+    return pv, pf, tk, s, mv
+
+
+def near_counts(margin_v, tau, perf, topk, index_base=0, rel=1e-6):
+    """Candidates whose V margin lies within 1e-6 of the validity cut tau
+    (absolute: tau is 0 at thr = 0.5) and survivors whose P score lies
+    within 1e-6 (relative) of the k-th kept score."""
+    near_tau = int(np.sum(np.abs(margin_v.astype(np.float64) - tau) <= rel * max(1.0, abs(tau))))
+    kept = topk[topk >= 0] - index_base
+    if kept.size == 0:
+        return near_tau, 0
+    kth = float(perf[kept[-1]])
+    finite = perf[np.isfinite(perf)].astype(np.float64)
+    near_k = int(np.sum(np.abs(finite - kth) <= rel * abs(kth)))
+    return near_tau, near_k
+
+
 def assert_same_bits(a, b, what, nan_equal=False):
     """Bit-for-bit equality of float32 arrays.  With nan_equal, a NaN matches
     any NaN: IEEE 754 leaves the bits of a NaN an operation generates to the
@@ -79,13 +120,3 @@ def assert_parity(gpu, orc):
     assert_same_bits(gpf, opf, "perf")
     assert_pvalid(gpv, opv)
     assert np.array_equal(gtk, otk), f"top-k differs: {gtk[:10]} vs {otk[:10]}"
-
-
-def topk_from_scores(perf, k, index_base=0):
-    """First k of the full order (score desc, index asc) over finite scores."""
-    idx = np.nonzero(perf > -np.inf)[0]
-    order = idx[np.lexsort((idx, -perf[idx].astype(np.float64)))]
-    out = np.full(k, -1, np.int64)
-    m = min(k, order.size)
-    out[:m] = order[:m] + index_base
-    return out, idx.size
