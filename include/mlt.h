@@ -258,6 +258,22 @@ int mlt_sa_step(void *stream, const int32_t *radices, const float *option_values
                 int64_t m, float temperature, float thr, int64_t *out_next,
                 float *out_next_score, int32_t *out_accepted);
 
+/* Cross-rank merge of kept candidates (Sec. 2: the explorer keeps the
+ * (alpha+1)N configurations model P ranks highest; with the batch sharded
+ * over G ranks, each rank's top-k is gathered and merged): writes to
+ * out_topk the k best of the m pairs (scores[i], indices[i]) by the
+ * screening's own order -- P score descending (-0 equal to +0), then
+ * global candidate index ascending -- padded with -1.
+ *   scores   device [m] fp32 (finite for a kept candidate)
+ *   indices  device [m] int64 global candidate indices; a negative index
+ *            marks an empty slot (ignored); the others must be distinct
+ *   m        0 .. 262,144 (for example G ranks x k)
+ *   k        1 .. 16,384
+ *   out_topk device [k] int64
+ * Asynchronous on `stream`. */
+int mlt_merge_topk(void *stream, const float *scores, const int64_t *indices, int64_t m, int k,
+                   int64_t *out_topk);
+
 /* Model A rerank (Sec. 2, "Hidden Feature Extractor & ML Model A"): from the
  * (alpha+1)N candidates kept by screening, model A -- a performance
  * regressor over visible and hidden features, typically deeper than P
@@ -372,18 +388,27 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  * trees (0 in any field = let the library choose it):
  *   candidates   candidates per CTA: a multiple of 32, 32 .. 256
  *   splits       threads sharing one candidate's trees: 1, 2 or 4 for
- *                ensembles of depth <= 10 (groups of warps, leaves summed
- *                in tree order through shared memory), 1, 2, 4 or 8 for
- *                deeper ones (lanes of a warp, summed through shuffles);
- *                candidates x splits <= 256
+ *                ensembles of depth <= 10 and split tables (groups of
+ *                warps, leaves summed in tree order through shared
+ *                memory), 1, 2, 4 or 8 for compact tables (lanes of a
+ *                warp, summed through shuffles); candidates x splits <= 256
+ *                (<= 512 for split tables)
  *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10),
  *                4 or 8 (deeper)
- *   chunk_trees  trees per shared-memory chunk, 1, 2, 4, 8 or 16 (depth
- *                <= 10 only)
- *   nbuf         chunk buffers, 2 or 3 (depth <= 10 only)
+ *   chunk_trees  trees per shared-memory chunk, 1, 2, 4, 8 or 16 (full,
+ *                half and split tables)
+ *   nbuf         chunk buffers, 2 or 3 (full, half and split tables)
  * A shape that does not fit shared memory falls back to the library's
  * choice.  Results never depend on the shape.  Host-only. */
 int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf);
+
+/* Tuning: the table format of models V and P deeper than 10 levels, for
+ * ensembles loaded after this call.  levels = 6 (the default) or 7: a
+ * split table, whose first `levels` levels stream through shared memory
+ * with the tile while the deeper nodes are read from L2; 0: a compact
+ * table, read wholly through L1/L2.  Model A always uses the compact
+ * table.  Results never depend on the format.  Host-only. */
+int mlt_tune_head_levels(int levels);
 
 /* Cumulative number of GPU kernels this library has launched. */
 int64_t mlt_kernel_launches(void);

@@ -51,6 +51,8 @@ using namespace mlt;
 
 thread_local std::string t_err;
 
+constexpr long long kMaxMergePairs = 16LL * kMaxK;  // 16 ranks' top-k lists
+
 int fail(int code, const char* fmt, ...) {
   char buf[512];
   va_list ap;
@@ -131,6 +133,7 @@ ShapeOverride g_shape[3];
 // failure-detection self-test, armed by mlt_selftest_walk_timeout: the next
 // full-table V pass makes CTA g_stall_cta wait on a barrier phase that
 // nothing completes, for g_stall_ns (one shot)
+int g_head_levels = kSplitHeadDefault;  // split tables for deep V and P models (0: compact tables)
 int g_stall_cta = -1;
 unsigned long long g_stall_ns = 0;
 
@@ -274,9 +277,10 @@ int check_models(int dev, bool decoded = false) {
 // estimate of the survivors.  Full-table tiles are balanced over the SMs.
 ScreenShape plan_for(const DeviceModel& dm, int F, long long n_eff, const ShapeOverride& ov, bool v_pass) {
   const bool half = dm.kind == kTableHalf;
-  ScreenShape s = dm.kind != kTableCompact
-                      ? plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov, half)
-                      : plan_compact(F, n_eff, sm_count(), smem_optin(), ov);
+  ScreenShape s = dm.kind == kTableCompact ? plan_compact(F, n_eff, sm_count(), smem_optin(), ov)
+                  : dm.kind == kTableSplit
+                      ? plan_split(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov)
+                      : plan_full(F, dm.n_trees, dm.tree_bytes, n_eff, sm_count(), smem_optin(), ov, half);
   if (s.threads == 0 && (ov.threads || ov.chunk_trees || ov.nbuf || ov.lanes || ov.group))
     return plan_for(dm, F, n_eff, ShapeOverride(), v_pass);
   // no more CTAs per SM than the plan counted on
@@ -489,6 +493,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   av.chunk_trees = sv.chunk_trees;
   av.nbuf = sv.nbuf;
   av.max_depth = V.depth;
+  av.tail = reinterpret_cast<const uint2*>(V.tail);
   // every call starts from a fresh selection state: its tickets decide which
   // CTA scans the tile counts and ranks the keys, so a count left behind by
   // an earlier call (one that stopped part-way) must not carry over
@@ -526,6 +531,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   ap.chunk_trees = sp.chunk_trees;
   ap.nbuf = sp.nbuf;
   ap.max_depth = P.depth;
+  ap.tail = reinterpret_cast<const uint2*>(P.tail);
   const long long tiles_p = (n + sp.threads - 1) / sp.threads;
   MLT_CUDA(dec ? launch_traverse_dec(P, ap, *dec, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
            "P pass launch");
@@ -629,6 +635,7 @@ int run_stream(cudaStream_t st, const float* feats, const DecodeParams* dec0, lo
     av.chunk_trees = sv.chunk_trees;
     av.nbuf = sv.nbuf;
     av.max_depth = V.depth;
+    av.tail = reinterpret_cast<const uint2*>(V.tail);
     const long long tiles_v = (nb + sv.threads - 1) / sv.threads;
     MLT_CUDA(dec0 ? launch_traverse_dec(V, av, d, sv, tiles_v, st) : launch_traverse(V, av, sv, tiles_v, st),
              "V pass launch");
@@ -641,6 +648,7 @@ int run_stream(cudaStream_t st, const float* feats, const DecodeParams* dec0, lo
     ap.chunk_trees = sp.chunk_trees;
     ap.nbuf = sp.nbuf;
     ap.max_depth = P.depth;
+    ap.tail = reinterpret_cast<const uint2*>(P.tail);
     const long long tiles_p = (nb + sp.threads - 1) / sp.threads;
     MLT_CUDA(dec0 ? launch_traverse_dec(P, ap, d, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
              "P pass launch");
@@ -673,6 +681,113 @@ int run_screen(cudaStream_t st, const float* feats, const DecodeParams* dec, lon
   const int rc = ensure_scratch(n);
   if (rc != MLT_OK) return rc;
   return run_screen_with(st, feats, dec, n, thr, k, out_pvalid, out_perf, out_topk, g_scr.s, true);
+}
+
+// Split table (kTableSplit, deep models V and P): validate like
+// pack_ensemble, then store each tree's first H levels and its level-H exits
+// as a head block and everything below level H as breadth-first compact
+// records in one tail array (layout in mlt_internal.cuh).
+int pack_split(const mlt_node* nodes, int n_trees, int depth, int F, int H, std::vector<unsigned char>& out,
+               DeviceModel& dm) {
+  {
+    std::vector<unsigned char> scratch;
+    DeviceModel probe;
+    const int rc = pack_ensemble(nodes, n_trees, depth, F, scratch, probe);  // validation
+    if (rc != MLT_OK) return rc;
+  }
+  const int slots = (2 << depth) - 1;
+  const uint32_t hb = split_head_bytes(H);
+  const int n_head = (1 << H) - 1;         // slots of levels 0 .. H-1
+  const int n_exit_end = (2 << H) - 1;     // level-H slots end here
+  const size_t tail_off = align16(static_cast<size_t>(n_trees) * hb);
+  std::vector<unsigned char> heads(tail_off, 0);
+  std::vector<uint32_t> recs;  // tail records, two words each
+  std::vector<unsigned char> reach(slots);
+  std::vector<float> inherit(n_exit_end);
+  std::vector<int> order;
+  auto split_meta = [](const mlt_node& nd, uint32_t left) {
+    return static_cast<uint32_t>(nd.feature) | (left << kCompactChildShift) |
+           (nd.default_left ? kMetaDefaultLeft : 0u);
+  };
+  for (int t = 0; t < n_trees; ++t) {
+    const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+    unsigned char* dst = heads.data() + static_cast<size_t>(t) * hb;
+    std::fill(reach.begin(), reach.end(), 0);
+    reach[0] = 1;
+    for (int j = 0; j < slots; ++j) {
+      if (reach[j] && tr[j].feature >= 0) {
+        reach[2 * j + 1] = 1;
+        reach[2 * j + 2] = 1;
+      }
+    }
+    for (int j = 0; j < n_exit_end; ++j) {
+      if (reach[j] && tr[j].feature == -1)
+        inherit[j] = tr[j].value;
+      else if (!reach[j])
+        inherit[j] = inherit[(j - 1) / 2];  // below a leaf: copy it down
+      else
+        inherit[j] = 0.0f;
+    }
+    // levels 0 .. H-1: splits, or pass-through records
+    for (int j = 0; j < n_head; ++j) {
+      const mlt_node& nd = tr[j];
+      const bool split = reach[j] && nd.feature >= 0;
+      const float thr = split ? nd.value : 0.0f;
+      const uint32_t meta = split ? (static_cast<uint32_t>(nd.feature) | (nd.default_left ? kMetaDefaultLeft : 0u)) : 0u;
+      std::memcpy(dst + 8 * j, &thr, 4);
+      std::memcpy(dst + 8 * j + 4, &meta, 4);
+    }
+    // level H: leaves, or split nodes whose children open the tail
+    const size_t base = recs.size() / 2;
+    if (base > 0xFFFFFFFFull) return fail(MLT_EINVAL, "split table too large");
+    order.clear();
+    for (int j = n_head; j < n_exit_end; ++j) {
+      const mlt_node& nd = tr[j];
+      float v;
+      uint32_t meta;
+      if (reach[j] && nd.feature >= 0) {
+        const uint32_t left = static_cast<uint32_t>(order.size());
+        order.push_back(2 * j + 1);
+        order.push_back(2 * j + 2);
+        v = nd.value;
+        meta = split_meta(nd, left);
+      } else {
+        v = inherit[j];
+        meta = kMetaLeaf;
+      }
+      std::memcpy(dst + 8 * j, &v, 4);
+      std::memcpy(dst + 8 * j + 4, &meta, 4);
+    }
+    const uint32_t b32 = static_cast<uint32_t>(base);
+    std::memcpy(dst + hb - 8, &b32, 4);
+    // below level H, breadth first (children adjacent)
+    for (size_t q = 0; q < order.size(); ++q) {
+      const mlt_node& nd = tr[order[q]];
+      uint32_t vb, meta;
+      std::memcpy(&vb, &nd.value, 4);
+      if (nd.feature >= 0) {
+        const uint32_t left = static_cast<uint32_t>(order.size());
+        if (left > kCompactChildMask) return fail(MLT_EINVAL, "tree %d has too many nodes", t);
+        order.push_back(2 * order[q] + 1);
+        order.push_back(2 * order[q] + 2);
+        meta = split_meta(nd, left);
+      } else {
+        meta = kMetaLeaf;
+      }
+      recs.push_back(vb);
+      recs.push_back(meta);
+    }
+  }
+  out.assign(tail_off + recs.size() * 4, 0);
+  std::memcpy(out.data(), heads.data(), heads.size());
+  if (!recs.empty()) std::memcpy(out.data() + tail_off, recs.data(), recs.size() * 4);
+  dm.kind = kTableSplit;
+  dm.n_trees = n_trees;
+  dm.depth = depth;
+  dm.tree_bytes = hb;
+  dm.head_levels = H;
+  dm.tail_off = tail_off;
+  return MLT_OK;
 }
 
 // Half table (kTableHalf): validate like pack_ensemble, then store the
@@ -764,6 +879,7 @@ int install_model(int model_id, const std::vector<unsigned char>& packed, const 
   m.dm = dm;
   m.dm.table = d;
   m.dm.bytes = packed.size();
+  if (dm.kind == kTableSplit) m.dm.tail = d + dm.tail_off;
   return MLT_OK;
 }
 
@@ -789,9 +905,21 @@ int mlt_load_ensemble(int model_id, const mlt_node* nodes, int n_trees, int dept
   if (g_F <= 0) return fail(MLT_EINVAL, "call mlt_set_num_features before loading ensembles");
   std::vector<unsigned char> packed;
   DeviceModel dm;
-  int rc = pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
+  // models V and P deeper than a full table: split tables (model A keeps
+  // the compact table its rerank walks)
+  const bool split = depth > kMaxFullDepth && model_id != MLT_MODEL_A && g_head_levels > 0;
+  int rc = split ? pack_split(nodes, n_trees, depth, g_F, g_head_levels, packed, dm)
+                 : pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
   if (rc != MLT_OK) return rc;
   return install_model(model_id, packed, dm);
+}
+
+int mlt_tune_head_levels(int levels) {
+  if (!(levels == 0 || levels == 6 || levels == 7))
+    return fail(MLT_EINVAL, "levels must be 0 (compact tables), 6 or 7, got %d", levels);
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_head_levels = levels;
+  return MLT_OK;
 }
 
 int mlt_load_ensemble_f16(int model_id, const mlt_node* nodes, int n_trees, int depth) {
@@ -858,6 +986,19 @@ int mlt_screen_noalloc(void* stream, const float* feats, int64_t n, float thr, i
   // cleared at the start of the sequence, the error word only when
   // mlt_sync_status reads it (so a fault of this call stays visible)
   return run_screen_with(st, feats, nullptr, n, thr, k, out_pvalid, out_perf, out_topk, s, false);
+}
+
+int mlt_merge_topk(void* stream, const float* scores, const int64_t* indices, int64_t m, int k,
+                   int64_t* out_topk) {
+  if (m < 0 || m > kMaxMergePairs) return fail(MLT_EINVAL, "m must lie in [0, %lld], got %lld", kMaxMergePairs,
+                                               static_cast<long long>(m));
+  if (k < 1 || k > kMaxK) return fail(MLT_EINVAL, "k must lie in [1, %d], got %d", kMaxK, k);
+  if ((m > 0 && (scores == nullptr || indices == nullptr)) || out_topk == nullptr)
+    return fail(MLT_EINVAL, "device buffers must be non-NULL");
+  MLT_CUDA(launch_merge_topk(scores, indices, m, k, out_topk, static_cast<cudaStream_t>(stream)), "merge launch");
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_launches += m > 0 ? 1 : 0;
+  return MLT_OK;
 }
 
 int mlt_screen_until(void* stream, const float* feats, int64_t n_total, int64_t batch, int64_t target, float thr,
@@ -1311,8 +1452,8 @@ int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk
         chunk_trees == 16))
     return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8 or 16");
   if (!(nbuf == 0 || nbuf == 2 || nbuf == 3)) return fail(MLT_EINVAL, "nbuf must be 0, 2 or 3");
-  if (candidates && splits && candidates * splits > 256)
-    return fail(MLT_EINVAL, "candidates x splits must be at most 256");
+  if (candidates && splits && candidates * splits > 512)
+    return fail(MLT_EINVAL, "candidates x splits must be at most 512");
   std::lock_guard<std::mutex> lk(g_mu);
   ShapeOverride& o = g_shape[model_id];
   o.threads = candidates;

@@ -62,7 +62,28 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 //                      (binary16)}.
 // The features are rounded to binary16 when staged, so a candidate is
 // compared and scored exactly as the rounded model scores the rounded row.
-enum TableKind : int { kTableFull = 0, kTableCompact = 1, kTableHalf = 2 };
+//
+// Split table (models V and P deeper than kMaxFullDepth): each tree's first
+// H levels as a complete heap that streams through shared memory like a
+// full table, and the rest as compact records read from global memory:
+//   head block (split_head_bytes(H) bytes, one per tree, contiguous):
+//     heap slots 0 .. 2^H - 2 (levels 0 .. H-1): 8-byte {threshold, meta}
+//       with meta = feature | NaN-left bit (bit 31); a slot on or below a
+//       shallower leaf is a pass-through {0, 0} (every exit below it holds
+//       that leaf, so the direction taken does not matter);
+//     heap slots 2^H - 1 .. 2^(H+1) - 2 (level H, the exits): a leaf
+//       {value, kMetaLeaf} or the level-H split node itself in the compact
+//       format, its child index counted from the tree's tail base;
+//     last 8 bytes: {tail base (record index into the tail array), 0};
+//   tail array (after the n_trees head blocks, 16-byte aligned): every
+//     tree's nodes below level H in breadth-first order, compact records
+//     (children adjacent, right = left + 1).
+// The walk reads H levels and the exit from shared memory; only paths that
+// go deeper than H touch global memory (L2-resident: evict_last).
+enum TableKind : int { kTableFull = 0, kTableCompact = 1, kTableHalf = 2, kTableSplit = 3 };
+
+constexpr int kSplitHeadDefault = 6;  // head levels of a split table (6 or 7)
+__host__ __device__ constexpr uint32_t split_head_bytes(int H) { return (2u << H) * 8u; }
 
 struct HalfLayout {
   uint32_t n_inner;   // nodes in levels [0, D-1)
@@ -114,7 +135,10 @@ struct DeviceModel {
   int kind = kTableFull;
   int n_trees = 0;
   int depth = 0;
-  uint32_t tree_bytes = 0;  // full tables
+  uint32_t tree_bytes = 0;  // full and half tables: bytes per tree; split tables: head block bytes
+  int head_levels = 0;      // split tables: H
+  const unsigned char* tail = nullptr;  // split tables: the tail records
+  size_t tail_off = 0;                  // split tables: byte offset of the tail records
 };
 
 // ---------------------------------------------------------------------------
@@ -194,7 +218,8 @@ struct TraverseArgs {
   uint32_t tree_bytes;     // full table
   int chunk_trees;         // full table: trees per shared-memory chunk
   int nbuf;                // full table: chunk buffers
-  int max_depth;           // compact table
+  int max_depth;           // compact and split tables
+  const uint2* tail;       // split tables: the tail records
   float tau;
   // outputs
   float* out_pvalid;
@@ -260,6 +285,10 @@ FullKernelPtr full_kernel_sf(int depth, int group);
 FullDecKernelPtr full_dec_kernel_sf(int depth, int group);
 // traverse_half.cu: half tables (one tree group, stored features only)
 FullKernelPtr half_kernel(int depth, int group, bool sync_free);
+// traverse_split.cu: split tables, H head levels, q tree groups (0: one
+// group, barrier-free pipeline), G in {4, 8}
+FullKernelPtr split_kernel(int head_levels, int group, int q);
+FullDecKernelPtr split_dec_kernel(int head_levels, int group, int q);
 
 // traverse.cu
 // n_eff: candidates the pass is expected to walk (used for load balance).
@@ -268,6 +297,9 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tree_bytes, long long n_eff, 
                       int device_smem_optin, const ShapeOverride& ov, bool half);
 ScreenShape plan_compact(int F, long long n_eff, int sms, int device_smem_optin,
                          const ShapeOverride& ov);
+// split tables: head blocks of hb bytes
+ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms, int device_smem_optin,
+                       const ShapeOverride& ov);
 // Pad a full-table shape's shared memory so that at most s.resident CTAs fit
 // on an SM.
 ScreenShape cap_residency(const ScreenShape& s, int optin);
@@ -311,6 +343,9 @@ cudaError_t launch_compact(const Scratch& s, long long n, int tile, long long n_
 // count: survivors to select from (null: the batch's own count)
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base,
                         int64_t* out_topk, int sms, const unsigned* count, cudaStream_t st);
+// the k best of m (score, global index) pairs (cross-rank merge)
+cudaError_t launch_merge_topk(const float* scores, const int64_t* idx, long long m, int k, int64_t* out,
+                              cudaStream_t st);
 cudaError_t launch_accumulate(StreamState* ss, const SelectState* st_, long long n_batch,
                               unsigned target, cudaStream_t st);
 cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaStream_t st);

@@ -325,6 +325,63 @@ cudaError_t launch_stream_stats(const StreamState* ss, int64_t* out_stats, cudaS
   return launch_pdl(k_stream_stats, dim3(1), dim3(32), 0, st, ss, out_stats);
 }
 
+namespace {
+
+constexpr int kMergeThreads = 256;
+constexpr int kMergeTile = 1024;  // pairs staged in shared memory per pass
+
+// Order-preserving unsigned image of a score (-0 folded onto +0), the high
+// word of the screening's rank keys.
+__device__ __forceinline__ uint32_t mono_score(float s) {
+  const uint32_t u = __float_as_uint(s == 0.0f ? 0.0f : s);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Rank of every pair (score, global index) among the m pairs by (score
+// descending, index ascending), counted as the number of better pairs
+// (indices are unique, so ranks are too); pair i of rank r < k goes to
+// out[r].  Pairs with a negative index are empty slots: never ranked,
+// never counted.
+__global__ void __launch_bounds__(kMergeThreads)
+    k_merge_rank(const float* scores, const int64_t* idx, long long m, int k, int64_t* out) {
+  __shared__ uint32_t s_key[kMergeTile];
+  __shared__ long long s_idx[kMergeTile];
+  const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool mine = i < m && idx[i] >= 0;
+  const uint32_t key = mine ? mono_score(scores[i]) : 0u;
+  const long long id = mine ? static_cast<long long>(idx[i]) : 0;
+  long long rank = 0;
+  for (long long j0 = 0; j0 < m; j0 += kMergeTile) {
+    const int len = static_cast<int>(min(static_cast<long long>(kMergeTile), m - j0));
+    __syncthreads();
+    for (int t = threadIdx.x; t < len; t += blockDim.x) {
+      const long long jj = idx[j0 + t];
+      s_key[t] = jj >= 0 ? mono_score(scores[j0 + t]) : 0u;
+      s_idx[t] = jj;  // negative: an empty slot
+    }
+    __syncthreads();
+    if (mine)
+      for (int t = 0; t < len; ++t) {
+        const uint32_t kj = s_key[t];
+        const long long ij = s_idx[t];
+        rank += (ij >= 0) & ((kj > key) | ((kj == key) & (ij < id)));
+      }
+  }
+  if (mine && rank < k) out[rank] = id;
+}
+
+}  // namespace
+
+cudaError_t launch_merge_topk(const float* scores, const int64_t* idx, long long m, int k, int64_t* out,
+                              cudaStream_t st) {
+  // every slot starts empty (-1: all bits set)
+  cudaError_t e = cudaMemsetAsync(out, 0xFF, sizeof(int64_t) * static_cast<size_t>(k), st);
+  if (e != cudaSuccess || m <= 0) return e;
+  const long long blocks = (m + kMergeThreads - 1) / kMergeThreads;
+  k_merge_rank<<<static_cast<unsigned>(blocks), kMergeThreads, 0, st>>>(scores, idx, m, k, out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_topk(const Scratch& s, long long n, int k, long long index_base, int64_t* out_topk, int sms,
                         const unsigned* count, cudaStream_t st) {
   int n2k = 2;

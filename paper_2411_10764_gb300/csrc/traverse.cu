@@ -117,6 +117,67 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
   return best;  // threads == 0: nothing fits
 }
 
+// Split table (deep trees): the same tile and chunk pipeline as a full
+// table, streaming head blocks of hb bytes; the paths that leave the head
+// wait on L2, so the shape maximises the walks in flight per SM
+// (resident CTAs x candidates x tree groups x trees per thread), counted up
+// to kSplitSaturation, per candidate of the busiest SM.  Ties go to larger
+// tiles (each tile re-streams every head block), then to fewer tree groups.
+// Up to 512 threads per CTA (the split kernels' launch bound).
+ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms, int optin,
+                       const ShapeOverride& ov) {
+  constexpr double kSplitSaturation = 4096.0;
+  if (sms < 1) sms = 1;
+  if (n_eff < 1) n_eff = 1;
+  ScreenShape best{};
+  double best_cost = 1e300;
+  for (int q : {1, 2, 4}) {
+    if (ov.lanes && q != ov.lanes) continue;
+    for (int tc : {256, 128, 64, 32}) {
+      if (ov.threads && tc != ov.threads) continue;
+      if (tc * q > 512) continue;
+      for (int ch : {16, 8, 4}) {
+        if (ov.chunk_trees && ch != ov.chunk_trees) continue;
+        const int chunk = std::min(ch, n_trees);
+        for (int nb : {2, 3}) {
+          if (ov.nbuf && nb != ov.nbuf) continue;
+          const size_t smem = full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * hb, q, chunk);
+          if (smem + kStaticSmem > static_cast<size_t>(optin)) continue;
+          for (int g : {8, 4}) {
+            if (ov.group && g != ov.group) continue;
+            if (g > std::max(4, chunk / q)) continue;  // a group's share of a chunk holds g trees
+            const int regs = g == 8 ? 88 : 64;
+            const long long tiles = (n_eff + tc - 1) / tc;
+            const long long tiles_sm = (tiles + sms - 1) / sms;
+            const int fit = static_cast<int>(std::min<size_t>(
+                {kSmPerSm / (smem + kStaticSmem + kCtaReserve), static_cast<size_t>(2048 / (tc * q)),
+                 static_cast<size_t>(65536 / (tc * q * regs)), 32}));
+            if (fit < 1) continue;
+            const int res = static_cast<int>(std::min<long long>(fit, tiles_sm));
+            const int gg = std::min(g, std::max(1, chunk / q));
+            const double inflight = static_cast<double>(res) * tc * q * gg;
+            const double cost = static_cast<double>(tiles_sm) * tc / std::min(inflight, kSplitSaturation) *
+                                (1.0 + 0.02 * q) * (1.0 + 32.0 / tc);
+            if (cost < best_cost * (1.0 - 1e-9)) {
+              best_cost = cost;
+              best.threads = tc;
+              best.lanes = q;
+              best.chunk_trees = chunk;
+              best.nbuf = nb;
+              best.group = g;
+              best.smem = smem;
+              best.p_grid = sms * std::max(1, res);
+              best.resident = std::max(1, res);
+              best.sync_free = q == 1 && best.resident == 1 ? 1 : 0;
+            }
+          }
+        }
+      }
+    }
+  }
+  return best;
+}
+
 ScreenShape cap_residency(const ScreenShape& s, int optin) {
   if (s.threads == 0 || s.resident < 1) return s;
   const size_t per_cta = kStaticSmem + kCtaReserve;
@@ -219,9 +280,11 @@ cudaError_t launch_traverse(const DeviceModel& m, const TraverseArgs& args, cons
   }
   const dim3 grid(static_cast<unsigned>(ctas));
   if (m.kind != kTableCompact) {
+    const int q = shape.sync_free ? 0 : shape.lanes;
     FullKernelPtr k = m.kind == kTableHalf
                           ? (shape.lanes == 1 ? half_kernel(m.depth, shape.group, shape.sync_free != 0) : nullptr)
-                          : full_kernel(m.depth, shape.group, shape.sync_free ? 0 : shape.lanes);
+                      : m.kind == kTableSplit ? split_kernel(m.head_levels, shape.group, q)
+                                              : full_kernel(m.depth, shape.group, q);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));

@@ -95,13 +95,15 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args, 
   TraverseArgs a = args;
   long long ctas = n_tiles;
   if (m.kind == kTableHalf) return cudaErrorInvalidValue;  // half tables need stored features
-  if (args.p_pass && m.kind == kTableFull && shape.p_grid > 0) {
+  if (args.p_pass && (m.kind == kTableFull || m.kind == kTableSplit) && shape.p_grid > 0) {
     a.p_wave = shape.p_grid;
     ctas = (n_tiles + shape.p_grid - 1) / shape.p_grid * shape.p_grid;
   }
   const dim3 grid(static_cast<unsigned>(ctas));
-  if (m.kind == kTableFull) {
-    FullDecKernelPtr k = full_dec_kernel(m.depth, shape.group, shape.sync_free ? 0 : shape.lanes);
+  if (m.kind == kTableFull || m.kind == kTableSplit) {
+    const int q = shape.sync_free ? 0 : shape.lanes;
+    FullDecKernelPtr k = m.kind == kTableSplit ? split_dec_kernel(m.head_levels, shape.group, q)
+                                               : full_dec_kernel(m.depth, shape.group, q);
     if (k == nullptr) return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(shape.smem));

@@ -629,6 +629,88 @@ __device__ __forceinline__ float walk_chunk_half(uint32_t tb, int nt, uint32_t t
   return acc;
 }
 
+// ---------------------------------------------------------------------------
+// Split-table walk (deep trees: a shared-memory head, a global-memory tail)
+// ---------------------------------------------------------------------------
+// Walk trees q, q + Q, ... (< nt) of a chunk of head blocks at shared
+// address tb (head_bytes apart): H levels of 8-byte records and the exit
+// record from shared memory, then -- only where the exit is a split node --
+// the tail records from global memory (`tails`, kept in L2 with
+// evict_last), at most tail_steps of them.  The G walks of a thread issue
+// their tail loads together, and a warp stops once all its walks sit on a
+// leaf.  Q == 1: leaves added to acc in tree order; Q > 1: leaf t parked at
+// la + t * row_bytes for group 0's in-order sum.
+template <int H, int G, bool NANP, int Q>
+__device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, uint32_t head_bytes, uint32_t xa,
+                                                  uint32_t row_bytes, float acc, uint32_t la, const uint2* tails,
+                                                  int tail_steps) {
+  const unsigned long long keep = policy_evict_last();
+  for (int t = q; t < nt; t += G * Q) {
+    uint32_t base[G], j[G];
+    bool in[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      in[g] = t + g * Q < nt;
+      base[g] = tb + static_cast<uint32_t>(in[g] ? t + g * Q : t) * head_bytes;
+      j[g] = 0;
+    }
+#pragma unroll
+    for (int l = 0; l < H; ++l) {
+      uint2 r[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) r[g] = lds_u2(base[g] + j[g] * 8u);
+      float x[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
+#pragma unroll
+      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], r[g].x, r[g].y);
+    }
+    // the exit record (level H) and the tree's tail base
+    uint2 r[G];
+    uint32_t tbase[G];
+    bool live[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      r[g] = lds_u2(base[g] + j[g] * 8u);
+      tbase[g] = lds_u32(base[g] + head_bytes - 8u);
+      live[g] = in[g] && !(r[g].y & kMetaLeaf);
+    }
+    bool any = false;
+#pragma unroll
+    for (int g = 0; g < G; ++g) any |= live[g];
+    for (int s = 0; s < tail_steps && __any_sync(0xFFFFFFFFu, any); ++s) {
+      uint32_t idx[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        idx[g] = 0;
+        if (live[g]) {
+          const float x = lds_f32((r[g].y & kCompactFeatureMask) * row_bytes + xa);
+          idx[g] = tbase[g] + ((r[g].y >> kCompactChildShift) & kCompactChildMask) + go_right<NANP>(x, r[g].x, r[g].y);
+        }
+      }
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+        if (live[g]) r[g] = ldg_u2_hint(tails + idx[g], keep);
+      any = false;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        live[g] = live[g] && !(r[g].y & kMetaLeaf);
+        any |= live[g];
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (!in[g]) continue;
+      const float leaf = __uint_as_float(r[g].x);
+      if (Q == 1)
+        acc += leaf;
+      else
+        sts_f32(la + static_cast<uint32_t>(t + g * Q) * row_bytes, leaf);
+    }
+  }
+  return acc;
+}
+
 // Even split of `len` items into `parts` contiguous pieces whose sizes
 // differ by at most one; piece i starts at split_start(len, parts, i).  The
 // survivor count is a 32-bit value, so 32-bit arithmetic suffices (a 64-bit
@@ -676,7 +758,9 @@ __device__ __forceinline__ void cta_tile(const TraverseArgs& a, long long count,
 // refills it, so warps drift up to nbuf - 1 chunks apart instead of meeting
 // at a CTA barrier per chunk.  That wins where one CTA holds the SM; with two
 // resident CTAs the barrier version keeps the refills further ahead.
-template <int D, int G, int QS, bool H = false>
+// SH > 0: a split table with SH head levels (tree_bytes = the head block;
+// D is unused).
+template <int D, int G, int QS, bool H = false, int SH = 0>
 __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const DecodeParams* dec) {
   constexpr int Q = QS == 0 ? 1 : QS;
   constexpr bool kSyncFree = QS == 0;
@@ -779,6 +863,11 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
       if constexpr (H)
         acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                   : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+      else if constexpr (SH > 0)
+        acc = nan ? walk_chunk_split<SH, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail,
+                                                     a.max_depth - SH)
+                  : walk_chunk_split<SH, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail,
+                                                      a.max_depth - SH);
       else
         acc = nan ? walk_chunk<D, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u)
                   : walk_chunk<D, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u);
@@ -827,6 +916,11 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     if constexpr (H)
       acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                 : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
+    else if constexpr (SH > 0)
+      acc = nan ? walk_chunk_split<SH, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail,
+                                                   a.max_depth - SH)
+                : walk_chunk_split<SH, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail,
+                                                    a.max_depth - SH);
     else
       acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
                 : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);

@@ -20,26 +20,14 @@ def shard_bounds(n: int, rank: int, world: int) -> tuple[int, int]:
     return n * rank // world, n * (rank + 1) // world
 
 
-def merge_topk(scores, indices, k: int) -> np.ndarray:
-    """Global top-k from the concatenated per-rank lists.
-
-    `indices` are global candidate indices (-1 marks an empty slot) and
-    `scores` their P scores.  Returns k indices, -1 padded."""
-    scores = np.asarray(scores, dtype=np.float32).reshape(-1)
-    indices = np.asarray(indices, dtype=np.int64).reshape(-1)
-    keep = indices >= 0
-    s, i = scores[keep], indices[keep]
-    order = np.lexsort((i, -s.astype(np.float64)))
-    out = np.full(int(k), -1, dtype=np.int64)
-    m = min(int(k), order.size)
-    out[:m] = i[order[:m]]
-    return out
-
-
-def gather_topk(local_indices, local_scores, k: int, group=None) -> np.ndarray:
+def gather_topk(local_indices, local_scores, k: int, group=None, merge=None):
     """Exchange every rank's local top-k and return the global top-k (on all
-    ranks).  Works with any torch.distributed backend; tensors live on the
-    backend's device (CPU for gloo, the current GPU for nccl)."""
+    ranks) as a numpy int64 array.  Works with any torch.distributed backend;
+    the exchanged tensors live on the backend's device (CPU for gloo, the
+    current GPU for nccl).  The merge runs in the library on the current GPU
+    (mlt_merge_topk: score descending, then global index ascending, -1
+    padded); `merge(scores, indices, k)` replaces it where no GPU is present
+    (the CPU multi-process tests)."""
     import torch
     import torch.distributed as dist
 
@@ -56,7 +44,12 @@ def gather_topk(local_indices, local_scores, k: int, group=None) -> np.ndarray:
     all_sc = [torch.empty_like(sc) for _ in range(world)]
     dist.all_gather(all_idx, idx, group=group)
     dist.all_gather(all_sc, sc, group=group)
-    return merge_topk(torch.cat(all_sc).cpu().numpy(), torch.cat(all_idx).cpu().numpy(), k)
+    cat_sc, cat_idx = torch.cat(all_sc), torch.cat(all_idx)
+    if merge is not None:
+        return np.asarray(merge(cat_sc.cpu().numpy(), cat_idx.cpu().numpy(), int(k)), dtype=np.int64)
+    gpu = torch.device("cuda", torch.cuda.current_device())
+    top = mlt.merge_topk(cat_sc.to(gpu), cat_idx.to(gpu), int(k))
+    return top.cpu().numpy()
 
 
 def screen_shard(feats_shard, thr: float, k: int, index_base: int, group=None, stream=None):

@@ -73,9 +73,11 @@ def lib(build_if_missing: bool = True):
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
+            "mlt_tune_head_levels": [i32],
             "mlt_walk_peak": [P, i32, P, i64, i32, P, P],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
+            "mlt_merge_topk": [P, P, P, i64, i32, P],
             "mlt_screen_until": [P, P, i64, i64, i64, f32, i32, P, P, P, P],
             "mlt_screen_until_decoded": [P, P, P, i32, P, i64, i64, i64, i64, f32, i32, P, P, P, P],
             "mlt_sa_step": [P, P, P, i32, P, P, P, P, P, P, i64, f32, f32, P, P, P],
@@ -266,6 +268,24 @@ def rerank(feats, cand, n_final: int, out_score=None, out_final=None, stream=Non
     return out_score, out_final
 
 
+def merge_topk(scores, indices, k: int, out=None, stream=None):
+    """mlt_merge_topk: the k best (score, global index) pairs (CUDA fp32 and
+    int64 tensors of equal length; a negative index is an empty slot) by
+    (score desc, index asc), -1 padded: returns a CUDA int64 tensor [k]."""
+    import torch
+
+    for t, dt in ((scores, torch.float32), (indices, torch.int64)):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t.dtype == dt and t.is_contiguous()):
+            raise TypeError("scores / indices must be contiguous float32 / int64 CUDA tensors")
+    m = indices.numel()
+    if scores.numel() != m:
+        raise ValueError("scores and indices differ in length")
+    if out is None:
+        out = torch.empty(int(k), dtype=torch.int64, device=indices.device)
+    _check(lib().mlt_merge_topk(_stream_ptr(stream), _dptr(scores), _dptr(indices), m, int(k), _dptr(out)))
+    return out
+
+
 def screen_host(feats: np.ndarray, thr: float, k: int, out=None, stream=None):
     """Screen a host [n][F] float32 array (copies in and out inside the call).
 
@@ -406,6 +426,12 @@ def tune_walk(model_id: int, candidates: int = 0, splits: int = 0, group: int = 
     """Fix (or with zeros, release) the tree walk's launch shape for one model."""
     _check(lib().mlt_tune_walk(int(model_id), int(candidates), int(splits), int(group), int(chunk_trees),
                                int(nbuf)))
+
+
+def tune_head_levels(levels: int) -> None:
+    """Table format of deep (depth > 10) V and P models loaded afterwards:
+    6 or 7 head levels in shared memory (split table), or 0 (compact)."""
+    _check(lib().mlt_tune_head_levels(int(levels)))
 
 
 def kernel_launches() -> int:

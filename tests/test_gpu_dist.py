@@ -45,3 +45,31 @@ def test_two_gpu_processes_shard_and_merge():
         assert top == want.tolist()
         a, b = D.shard_bounds(n, r, world)
         assert np.array_equal(np.array(perf_bits, np.uint32), pf[a:b].view(np.uint32))
+
+
+def _merge_case(rng, m, k, pad_frac=0.2, tie_frac=0.3):
+    scores = rng.normal(size=m).astype(np.float32)
+    ties = rng.random(m) < tie_frac
+    scores[ties] = np.float32(0.5)  # many equal scores: order by global index
+    scores[rng.random(m) < 0.05] = np.float32(-0.0)
+    scores[rng.random(m) < 0.05] = np.float32(0.0)
+    idx = rng.choice(1 << 40, size=m, replace=False).astype(np.int64)  # distinct, past 2^32
+    idx[rng.random(m) < pad_frac] = -1
+    return scores, idx
+
+
+@pytest.mark.parametrize("m,k", [(0, 5), (1, 1), (7, 20), (2048, 1024), (8 * 1024, 1024), (16 * 2048, 2048),
+                                 (5000, 16384), (262144, 64)])
+def test_device_merge_matches_the_oracle_order(m, k):
+    """mlt_merge_topk: the k best of m (score, global index) pairs by (score
+    desc, index asc), -0 equal to +0, empty slots skipped, -1 padded."""
+    import torch
+
+    from paper_2411_10764_gb300 import mlt
+    from dist_ranks import oracle_merge
+
+    rng = np.random.default_rng(m + k)
+    scores, idx = _merge_case(rng, m, k)
+    got = mlt.merge_topk(torch.from_numpy(scores).cuda(), torch.from_numpy(idx).cuda(), k)
+    mlt.sync_status()
+    assert np.array_equal(got.cpu().numpy(), oracle_merge(scores, idx, k))

@@ -24,7 +24,7 @@ def _expected(key, w):
 @pytest.fixture(scope="module")
 def deep():
     """Workload 5's shape at 3,001 candidates: 1,000 / 2,000 unbalanced trees
-    of depth <= 12 on 256 features, 30 % missing values (compact tables)."""
+    of depth <= 12 on 256 features, 30 % missing values."""
     return W.make_workload(5, seed=3, n=3001)
 
 
@@ -58,22 +58,62 @@ DEEP_SHAPES = [(c, q, g) for c in (32, 64, 128, 256) for q in (1, 2, 4, 8) for g
 
 
 @pytest.mark.parametrize("cand,lanes,group", DEEP_SHAPES)
-def test_deep_walk_every_shape(deep, cand, lanes, group):
+def test_compact_walk_every_shape(deep, cand, lanes, group):
+    """Deep trees as compact tables (every node read through L1/L2)."""
     try:
+        mlt.tune_head_levels(0)
         _force(candidates=cand, splits=lanes, group=group)
         got = gpu_screen(deep)
     finally:
         _release()
+        mlt.tune_head_levels(6)
     assert_parity(got, _expected("deep", deep))
 
 
 @pytest.mark.parametrize("cand,lanes,group", [(32, 8, 4), (64, 4, 8), (128, 1, 8), (32, 2, 8)])
-def test_deep_walk_decoded_shapes(deep_decoded, cand, lanes, group):
+def test_compact_walk_decoded_shapes(deep_decoded, cand, lanes, group):
     try:
+        mlt.tune_head_levels(0)
         _force(candidates=cand, splits=lanes, group=group)
         got = gpu_screen(deep_decoded)
     finally:
         _release()
+        mlt.tune_head_levels(6)
+    assert_parity(got, _expected("deep_decoded", deep_decoded))
+
+
+# split tables: (head levels, candidates per CTA, tree groups, trees in
+# flight, chunk, buffers); 256 features leave room for at most 128
+# candidates (F = 256) -- larger tiles fall back to the planner's choice
+SPLIT_TABLE_SHAPES = ([(6, c, q, g, 8, 2) for c in (32, 64, 128) for q in (1, 2, 4) for g in (4, 8)] +
+                      [(6, 64, 2, 4, ch, nb) for ch in (4, 16) for nb in (2, 3)] +
+                      [(7, c, q, g, ch, 2) for c, q, g, ch in ((128, 4, 4, 16), (64, 2, 8, 16), (32, 1, 4, 4),
+                                                               (128, 1, 8, 8))])
+
+
+@pytest.mark.parametrize("head,cand,groups,group,chunk,nbuf", SPLIT_TABLE_SHAPES)
+def test_split_walk_every_shape(deep, head, cand, groups, group, chunk, nbuf):
+    """Deep trees as split tables: the first `head` levels stream through
+    shared memory, deeper nodes come from L2."""
+    try:
+        mlt.tune_head_levels(head)
+        _force(candidates=cand, splits=groups, group=group, chunk_trees=chunk, nbuf=nbuf)
+        got = gpu_screen(deep)
+    finally:
+        _release()
+        mlt.tune_head_levels(6)
+    assert_parity(got, _expected("deep", deep))
+
+
+@pytest.mark.parametrize("head,cand,groups,group", [(6, 128, 4, 4), (6, 64, 1, 8), (7, 32, 2, 8), (7, 128, 2, 4)])
+def test_split_walk_decoded_shapes(deep_decoded, head, cand, groups, group):
+    try:
+        mlt.tune_head_levels(head)
+        _force(candidates=cand, splits=groups, group=group, chunk_trees=8, nbuf=2)
+        got = gpu_screen(deep_decoded)
+    finally:
+        _release()
+        mlt.tune_head_levels(6)
     assert_parity(got, _expected("deep_decoded", deep_decoded))
 
 
