@@ -388,13 +388,13 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  * trees (0 in any field = let the library choose it):
  *   candidates   candidates per CTA: a multiple of 32, 32 .. 256
  *   splits       threads sharing one candidate's trees: 1, 2 or 4 for
- *                ensembles of depth <= 10 and split tables (groups of
- *                warps, leaves summed in tree order through shared
- *                memory), 1, 2, 4 or 8 for compact tables (lanes of a
- *                warp, summed through shuffles); candidates x splits <= 256
- *                (<= 512 for split tables)
- *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10),
- *                4 or 8 (deeper)
+ *                ensembles of depth <= 10, 1, 2, 4 or 8 for split tables
+ *                (groups of warps, leaves summed in tree order through
+ *                shared memory), 1, 2, 4 or 8 for compact tables (lanes of
+ *                a warp, summed through shuffles); candidates x splits <=
+ *                256 (<= 512 for split tables, 1,024 with 8 groups)
+ *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10 and
+ *                split tables), 4 or 8 (compact tables)
  *   chunk_trees  trees per shared-memory chunk, 1, 2, 4, 8 or 16 (full,
  *                half and split tables)
  *   nbuf         chunk buffers, 2 or 3 (full, half and split tables)

@@ -705,12 +705,38 @@ int pack_split(const mlt_node* nodes, int n_trees, int depth, int F, int H, std:
   std::vector<unsigned char> reach(slots);
   std::vector<float> inherit(n_exit_end);
   std::vector<int> order;
-  auto split_meta = [](const mlt_node& nd, uint32_t left) {
-    return static_cast<uint32_t>(nd.feature) | (left << kCompactChildShift) |
-           (nd.default_left ? kMetaDefaultLeft : 0u);
+  // every node sends a missing value right: a node whose missing values go
+  // left is stored with its subtrees swapped, the negate bit (31) set and
+  // threshold -prev(t), so that "x < t or x missing" (its old left side) is
+  // "-x >= -prev(t) or -x missing" (its new right side)
+  std::vector<mlt_node> tn(slots);
+  std::vector<unsigned char> neg(slots);
+  std::vector<std::pair<int, int>> stack;
+  auto split_meta = [&](int j, uint32_t left) {
+    return static_cast<uint32_t>(tn[j].feature) | (left << kCompactChildShift) | (neg[j] ? kMetaDefaultLeft : 0u);
   };
   for (int t = 0; t < n_trees; ++t) {
-    const mlt_node* tr = nodes + static_cast<size_t>(t) * slots;
+    const mlt_node* orig = nodes + static_cast<size_t>(t) * slots;
+    for (mlt_node& nd : tn) nd = mlt_node{-2, 0.0f, 0, {0, 0, 0}};
+    std::fill(neg.begin(), neg.end(), 0);
+    stack.assign(1, {0, 0});
+    while (!stack.empty()) {
+      const auto [j, jn] = stack.back();
+      stack.pop_back();
+      const mlt_node& nd = orig[j];
+      tn[jn] = nd;
+      if (nd.feature < 0) continue;
+      if (nd.default_left) {
+        tn[jn].value = -std::nextafterf(nd.value, -INFINITY);
+        neg[jn] = 1;
+        stack.push_back({2 * j + 1, 2 * jn + 2});
+        stack.push_back({2 * j + 2, 2 * jn + 1});
+      } else {
+        stack.push_back({2 * j + 1, 2 * jn + 1});
+        stack.push_back({2 * j + 2, 2 * jn + 2});
+      }
+    }
+    const mlt_node* tr = tn.data();
     unsigned char* dst = heads.data() + static_cast<size_t>(t) * hb;
     std::fill(reach.begin(), reach.end(), 0);
     reach[0] = 1;
@@ -733,7 +759,7 @@ int pack_split(const mlt_node* nodes, int n_trees, int depth, int F, int H, std:
       const mlt_node& nd = tr[j];
       const bool split = reach[j] && nd.feature >= 0;
       const float thr = split ? nd.value : 0.0f;
-      const uint32_t meta = split ? (static_cast<uint32_t>(nd.feature) | (nd.default_left ? kMetaDefaultLeft : 0u)) : 0u;
+      const uint32_t meta = split ? (static_cast<uint32_t>(nd.feature) | (neg[j] ? kMetaDefaultLeft : 0u)) : 0u;
       std::memcpy(dst + 8 * j, &thr, 4);
       std::memcpy(dst + 8 * j + 4, &meta, 4);
     }
@@ -750,7 +776,7 @@ int pack_split(const mlt_node* nodes, int n_trees, int depth, int F, int H, std:
         order.push_back(2 * j + 1);
         order.push_back(2 * j + 2);
         v = nd.value;
-        meta = split_meta(nd, left);
+        meta = split_meta(j, left);
       } else {
         v = inherit[j];
         meta = kMetaLeaf;
@@ -770,7 +796,7 @@ int pack_split(const mlt_node* nodes, int n_trees, int depth, int F, int H, std:
         if (left > kCompactChildMask) return fail(MLT_EINVAL, "tree %d has too many nodes", t);
         order.push_back(2 * order[q] + 1);
         order.push_back(2 * order[q] + 2);
-        meta = split_meta(nd, left);
+        meta = split_meta(order[q], left);
       } else {
         meta = kMetaLeaf;
       }
@@ -1452,8 +1478,8 @@ int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk
         chunk_trees == 16))
     return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8 or 16");
   if (!(nbuf == 0 || nbuf == 2 || nbuf == 3)) return fail(MLT_EINVAL, "nbuf must be 0, 2 or 3");
-  if (candidates && splits && candidates * splits > 512)
-    return fail(MLT_EINVAL, "candidates x splits must be at most 512");
+  if (candidates && splits && candidates * splits > 1024)
+    return fail(MLT_EINVAL, "candidates x splits must be at most 1024");
   std::lock_guard<std::mutex> lk(g_mu);
   ShapeOverride& o = g_shape[model_id];
   o.threads = candidates;

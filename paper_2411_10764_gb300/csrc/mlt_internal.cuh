@@ -66,9 +66,13 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 // Split table (models V and P deeper than kMaxFullDepth): each tree's first
 // H levels as a complete heap that streams through shared memory like a
 // full table, and the rest as compact records read from global memory:
+//   every node sends a missing value right: a node whose missing values go
+//   left has its subtrees swapped, threshold -prev(t) and bit 31 of its meta
+//   set ("negate": the walk compares -x), so x < t (or missing) becomes
+//   -x >= -prev(t) (or missing), an unordered >= with no missing-value test;
 //   head block (split_head_bytes(H) bytes, one per tree, contiguous):
 //     heap slots 0 .. 2^H - 2 (levels 0 .. H-1): 8-byte {threshold, meta}
-//       with meta = feature | NaN-left bit (bit 31); a slot on or below a
+//       with meta = feature | negate bit (bit 31); a slot on or below a
 //       shallower leaf is a pass-through {0, 0} (every exit below it holds
 //       that leaf, so the direction taken does not matter);
 //     heap slots 2^H - 1 .. 2^(H+1) - 2 (level H, the exits): a leaf

@@ -118,24 +118,34 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
 }
 
 // Split table (deep trees): the same tile and chunk pipeline as a full
-// table, streaming head blocks of hb bytes; the paths that leave the head
-// wait on L2, so the shape maximises the walks in flight per SM
-// (resident CTAs x candidates x tree groups x trees per thread), counted up
-// to kSplitSaturation, per candidate of the busiest SM.  Ties go to larger
-// tiles (each tile re-streams every head block), then to fewer tree groups.
-// Up to 512 threads per CTA (the split kernels' launch bound).
+// table, streaming head blocks of hb bytes.  A warp's walk over a group of
+// trees lasts as long as its deepest path, which waits on one L2 round trip
+// per level below the head, so the shape maximises latency hiding per
+// candidate of the busiest SM.  Measured on GB300 (F = 256, 1,000-2,000
+// trees of depth <= 12): warps per SM count more than trees in flight per
+// thread (16 warps x 4 trees beat 8 warps x 8 trees by 1.24x), and a tree
+// group whose share of a chunk holds fewer than G trees wastes the rest
+// (8-tree chunks over 4 groups ran 1.7x slower than 16-tree chunks), and
+// two resident CTAs beat one CTA with the same warps (their chunk pipelines
+// do not meet at each other's barriers: 64 candidates x 8 groups x 2 CTAs
+// ran 8 % faster than 128 x 8 x 1).  The rule minimises
+//   tiles of the busiest SM x candidates per tile
+//     / (warps per SM x trees in flight per thread ^ 0.7)
+//     x (1 + 8 / tile) x (0.85 with two or more resident CTAs),
+// the tile factor for the head blocks every tile re-streams.  Up to 512
+// threads per CTA (1,024 with 8 tree groups: the split kernels' launch
+// bounds); registers (56-88 a thread) bound the warps an SM holds.
 ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms, int optin,
                        const ShapeOverride& ov) {
-  constexpr double kSplitSaturation = 4096.0;
   if (sms < 1) sms = 1;
   if (n_eff < 1) n_eff = 1;
   ScreenShape best{};
   double best_cost = 1e300;
-  for (int q : {1, 2, 4}) {
+  for (int q : {1, 2, 4, 8}) {
     if (ov.lanes && q != ov.lanes) continue;
     for (int tc : {256, 128, 64, 32}) {
       if (ov.threads && tc != ov.threads) continue;
-      if (tc * q > 512) continue;
+      if (tc * q > (q == 8 ? 1024 : 512)) continue;
       for (int ch : {16, 8, 4}) {
         if (ov.chunk_trees && ch != ov.chunk_trees) continue;
         const int chunk = std::min(ch, n_trees);
@@ -143,10 +153,10 @@ ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms
           if (ov.nbuf && nb != ov.nbuf) continue;
           const size_t smem = full_smem_bytes(F, tc, nb, static_cast<uint32_t>(chunk) * hb, q, chunk);
           if (smem + kStaticSmem > static_cast<size_t>(optin)) continue;
-          for (int g : {8, 4}) {
+          for (int g : {8, 4, 2}) {
             if (ov.group && g != ov.group) continue;
-            if (g > std::max(4, chunk / q)) continue;  // a group's share of a chunk holds g trees
-            const int regs = g == 8 ? 88 : 64;
+            if (!ov.group && g > std::max(2, chunk / q)) continue;  // idle tree slots
+            const int regs = g == 8 ? 88 : g == 4 ? 64 : 56;
             const long long tiles = (n_eff + tc - 1) / tc;
             const long long tiles_sm = (tiles + sms - 1) / sms;
             const int fit = static_cast<int>(std::min<size_t>(
@@ -154,10 +164,11 @@ ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms
                  static_cast<size_t>(65536 / (tc * q * regs)), 32}));
             if (fit < 1) continue;
             const int res = static_cast<int>(std::min<long long>(fit, tiles_sm));
-            const int gg = std::min(g, std::max(1, chunk / q));
-            const double inflight = static_cast<double>(res) * tc * q * gg;
-            const double cost = static_cast<double>(tiles_sm) * tc / std::min(inflight, kSplitSaturation) *
-                                (1.0 + 0.02 * q) * (1.0 + 32.0 / tc);
+            // tree groups with no tree of a chunk idle
+            const double warps = static_cast<double>(res) * tc * std::min(q, chunk) / 32.0;
+            const double gg = std::min(g, std::max(1, chunk / q));
+            const double cost = static_cast<double>(tiles_sm) * tc / (warps * std::pow(gg, 0.7)) * (1.0 + 8.0 / tc) *
+                                (res >= 2 ? 0.85 : 1.0) * (g > gg ? 1.05 : 1.0);
             if (cost < best_cost * (1.0 - 1e-9)) {
               best_cost = cost;
               best.threads = tc;

@@ -8,7 +8,7 @@ namespace mlt {
 namespace {
 
 template <int SH, int G, int QS>
-__global__ void __launch_bounds__(512, 1) k_traverse_split(const __grid_constant__ TraverseArgs a) {
+__global__ void __launch_bounds__(QS == 8 ? 1024 : 512, 1) k_traverse_split(const __grid_constant__ TraverseArgs a) {
   walk::traverse_full_body<1, G, QS, false, SH>(a, nullptr);
 }
 
@@ -19,13 +19,14 @@ FullKernelPtr split_for_q(int q) {
     case 1: return k_traverse_split<SH, G, 1>;
     case 2: return k_traverse_split<SH, G, 2>;
     case 4: return k_traverse_split<SH, G, 4>;
+    case 8: return k_traverse_split<SH, G, 8>;
     default: return nullptr;
   }
 }
 
 template <int SH>
 FullKernelPtr split_for_g(int g, int q) {
-  return g == 8 ? split_for_q<SH, 8>(q) : g == 4 ? split_for_q<SH, 4>(q) : nullptr;
+  return g == 8 ? split_for_q<SH, 8>(q) : g == 4 ? split_for_q<SH, 4>(q) : g == 2 ? split_for_q<SH, 2>(q) : nullptr;
 }
 
 }  // namespace

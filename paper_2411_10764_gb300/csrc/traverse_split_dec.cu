@@ -7,7 +7,7 @@ namespace mlt {
 namespace {
 
 template <int SH, int G, int QS>
-__global__ void __launch_bounds__(512, 1)
+__global__ void __launch_bounds__(QS == 8 ? 1024 : 512, 1)
     k_traverse_split_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
   walk::traverse_full_body<1, G, QS, false, SH>(a, &d);
 }
@@ -19,13 +19,15 @@ FullDecKernelPtr split_dec_for_q(int q) {
     case 1: return k_traverse_split_dec<SH, G, 1>;
     case 2: return k_traverse_split_dec<SH, G, 2>;
     case 4: return k_traverse_split_dec<SH, G, 4>;
+    case 8: return k_traverse_split_dec<SH, G, 8>;
     default: return nullptr;
   }
 }
 
 template <int SH>
 FullDecKernelPtr split_dec_for_g(int g, int q) {
-  return g == 8 ? split_dec_for_q<SH, 8>(q) : g == 4 ? split_dec_for_q<SH, 4>(q) : nullptr;
+  return g == 8 ? split_dec_for_q<SH, 8>(q) : g == 4 ? split_dec_for_q<SH, 4>(q)
+         : g == 2 ? split_dec_for_q<SH, 2>(q) : nullptr;
 }
 
 }  // namespace

@@ -640,7 +640,18 @@ __device__ __forceinline__ float walk_chunk_half(uint32_t tb, int nt, uint32_t t
 // their tail loads together, and a warp stops once all its walks sit on a
 // leaf.  Q == 1: leaves added to acc in tree order; Q > 1: leaf t parked at
 // la + t * row_bytes for group 0's in-order sum.
-template <int H, int G, bool NANP, int Q>
+// Split-table test: every node sends a missing value right.  A node whose
+// missing values go left is stored with its children swapped, bit 31 of its
+// meta set and threshold -prev(t) (prev(t) = the float below t): then
+// "x < t or x missing" (the old left side, now right) is exactly "-x >= -prev(t)
+// or -x missing" -- one sign flip and one unordered compare per visit, no
+// missing-value branch.
+__device__ __forceinline__ uint32_t go_right_split(float x, uint32_t thr_bits, uint32_t meta) {
+  const float xs = __uint_as_float(__float_as_uint(x) ^ (meta & 0x80000000u));
+  return !(xs < __uint_as_float(thr_bits)) ? 1u : 0u;
+}
+
+template <int H, int G, int Q>
 __device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, uint32_t head_bytes, uint32_t xa,
                                                   uint32_t row_bytes, float acc, uint32_t la, const uint2* tails,
                                                   int tail_steps) {
@@ -663,7 +674,7 @@ __device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, ui
 #pragma unroll
       for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
 #pragma unroll
-      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], r[g].x, r[g].y);
+      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right_split(x[g], r[g].x, r[g].y);
     }
     // the exit record (level H) and the tree's tail base
     uint2 r[G];
@@ -685,7 +696,7 @@ __device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, ui
         idx[g] = 0;
         if (live[g]) {
           const float x = lds_f32((r[g].y & kCompactFeatureMask) * row_bytes + xa);
-          idx[g] = tbase[g] + ((r[g].y >> kCompactChildShift) & kCompactChildMask) + go_right<NANP>(x, r[g].x, r[g].y);
+          idx[g] = tbase[g] + ((r[g].y >> kCompactChildShift) & kCompactChildMask) + go_right_split(x, r[g].x, r[g].y);
         }
       }
 #pragma unroll
@@ -864,10 +875,7 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
         acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                   : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
       else if constexpr (SH > 0)
-        acc = nan ? walk_chunk_split<SH, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail,
-                                                     a.max_depth - SH)
-                  : walk_chunk_split<SH, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail,
-                                                      a.max_depth - SH);
+        acc = walk_chunk_split<SH, G, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail, a.max_depth - SH);
       else
         acc = nan ? walk_chunk<D, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u)
                   : walk_chunk<D, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u);
@@ -917,10 +925,7 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
       acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                 : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
     else if constexpr (SH > 0)
-      acc = nan ? walk_chunk_split<SH, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail,
-                                                   a.max_depth - SH)
-                : walk_chunk_split<SH, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail,
-                                                    a.max_depth - SH);
+      acc = walk_chunk_split<SH, G, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail, a.max_depth - SH);
     else
       acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
                 : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);

@@ -131,7 +131,7 @@ def test_decoder_validation(L):
     assert call(r, prog, 0, 1, F=257) == -1
 
 
-@pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 128, 8, 4, 0, 0),
+@pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 256, 8, 4, 0, 0),
                                   (0, 64, 4, 3, 0, 0), (5, 64, 4, 4, 0, 0), (0, 0, 0, 0, 3, 0),
                                   (0, 0, 0, 0, 0, 4), (0, 288, 1, 4, 0, 0)])
 def test_walk_tuning_rejects(args):

@@ -88,7 +88,8 @@ def test_compact_walk_decoded_shapes(deep_decoded, cand, lanes, group):
 SPLIT_TABLE_SHAPES = ([(6, c, q, g, 8, 2) for c in (32, 64, 128) for q in (1, 2, 4) for g in (4, 8)] +
                       [(6, 64, 2, 4, ch, nb) for ch in (4, 16) for nb in (2, 3)] +
                       [(7, c, q, g, ch, 2) for c, q, g, ch in ((128, 4, 4, 16), (64, 2, 8, 16), (32, 1, 4, 4),
-                                                               (128, 1, 8, 8))])
+                                                               (128, 1, 8, 8), (128, 8, 2, 16), (32, 8, 2, 16))] +
+                      [(6, 64, 8, 4, 16, 3), (6, 128, 8, 2, 8, 2), (7, 128, 4, 2, 8, 3)])
 
 
 @pytest.mark.parametrize("head,cand,groups,group,chunk,nbuf", SPLIT_TABLE_SHAPES)
@@ -105,7 +106,8 @@ def test_split_walk_every_shape(deep, head, cand, groups, group, chunk, nbuf):
     assert_parity(got, _expected("deep", deep))
 
 
-@pytest.mark.parametrize("head,cand,groups,group", [(6, 128, 4, 4), (6, 64, 1, 8), (7, 32, 2, 8), (7, 128, 2, 4)])
+@pytest.mark.parametrize("head,cand,groups,group", [(6, 128, 4, 4), (6, 64, 1, 8), (7, 32, 2, 8), (7, 128, 2, 4),
+                                                    (7, 128, 8, 2)])
 def test_split_walk_decoded_shapes(deep_decoded, head, cand, groups, group):
     try:
         mlt.tune_head_levels(head)
