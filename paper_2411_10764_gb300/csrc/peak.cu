@@ -30,12 +30,11 @@ __global__ void __launch_bounds__(256)
   for (uint32_t i = tid; i < n16; i += blockDim.x) dst[i] = __ldg(src + i);
   const bool nan = __syncthreads_or(stage_row(a, nullptr, xs, nullptr, tile0, rows_here, TC));
   const uint32_t row_bytes = static_cast<uint32_t>(TC) * 4u;
-  const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(tid) * 4u;
-  const uint32_t tb = smem_u32(tbuf);
+  const unsigned char* xcol = reinterpret_cast<const unsigned char*>(xs) + static_cast<uint32_t>(tid) * 4u;
   float acc = 0.0f;
   for (int r = 0; r < rounds; ++r)
-    acc = nan ? walk_chunk<D, G, true, 1>(tb, 0, resident, a.tree_bytes, xa, row_bytes, acc, 0u)
-              : walk_chunk<D, G, false, 1>(tb, 0, resident, a.tree_bytes, xa, row_bytes, acc, 0u);
+    acc = nan ? walk_chunk<D, G, true, 1>(tbuf, 0, resident, a.tree_bytes, xcol, row_bytes, acc, 0u)
+              : walk_chunk<D, G, false, 1>(tbuf, 0, resident, a.tree_bytes, xcol, row_bytes, acc, 0u);
   if (tid < rows_here) out[tile0 + tid] = acc;
 }
 

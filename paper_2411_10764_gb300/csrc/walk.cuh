@@ -412,9 +412,19 @@ __device__ __forceinline__ void sts_f32(uint32_t a, float v) {
 // leaf t is parked at la + t * row_bytes for an in-order sum afterwards.
 // The 32-bit product meta * row_bytes drops meta's bit 31 because row_bytes
 // is a multiple of 2.
+// Shared-memory loads of the walk as ordinary C++ loads through pointers
+// derived from the kernel's shared array (so they compile to shared-memory
+// loads the compiler may schedule freely among the G walks); the mbarrier
+// waits around the walk carry a memory clobber, so no load moves across
+// them.
+template <typename T>
+__device__ __forceinline__ T ld_sm(const unsigned char* p, uint32_t off) {
+  return *reinterpret_cast<const T*>(p + off);
+}
+
 template <int D, int G, bool NANP, int Q>
-__device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t tree_bytes, uint32_t xa,
-                                            uint32_t row_bytes, float acc, uint32_t la) {
+__device__ __forceinline__ float walk_chunk(const unsigned char* tb, int q, int nt, uint32_t tree_bytes,
+                                            const unsigned char* xc, uint32_t row_bytes, float acc, uint32_t la) {
   constexpr FullLayout L = full_layout(D);
   // byte offsets folded with the heap index of each region's first node
   constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
@@ -423,7 +433,8 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
   constexpr uint32_t kLeaf = L.off_last + (1u << (D - 1)) * 8u - L.n_inner * 8u;
   int t = q;
   for (; t + (G - 1) * Q < nt; t += G * Q) {
-    uint32_t base[G], j[G];
+    const unsigned char* base[G];
+    uint32_t j[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       base[g] = tb + static_cast<uint32_t>(t + g * Q) * tree_bytes;
@@ -435,31 +446,32 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
       if (l < static_cast<int>(L.top)) {
 #pragma unroll
         for (int g = 0; g < G; ++g) {
-          const uint2 r = lds_u2(base[g] + j[g] * 8u);
+          const uint2 r = ld_sm<uint2>(base[g], j[g] * 8u);
           thr[g] = r.x;
           meta[g] = r.y;
         }
       } else {
 #pragma unroll
-        for (int g = 0; g < G; ++g) meta[g] = lds_u32(base[g] + kMeta + j[g] * 4u);
+        for (int g = 0; g < G; ++g) meta[g] = ld_sm<uint32_t>(base[g], kMeta + j[g] * 4u);
 #pragma unroll
-        for (int g = 0; g < G; ++g) thr[g] = lds_u32(base[g] + kThr + j[g] * 4u);
+        for (int g = 0; g < G; ++g) thr[g] = ld_sm<uint32_t>(base[g], kThr + j[g] * 4u);
       }
       float x[G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) x[g] = lds_f32(meta[g] * row_bytes + xa);
+      for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, meta[g] * row_bytes);
 #pragma unroll
       for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], thr[g], meta[g]);
     }
     uint2 r[G];
 #pragma unroll
-    for (int g = 0; g < G; ++g) r[g] = lds_u2(base[g] + kLast + j[g] * 8u);
+    for (int g = 0; g < G; ++g) r[g] = ld_sm<uint2>(base[g], kLast + j[g] * 8u);
     float x[G];
 #pragma unroll
-    for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
+    for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, r[g].y * row_bytes);
     float lf[G];
 #pragma unroll
-    for (int g = 0; g < G; ++g) lf[g] = lds_f32(base[g] + kLeaf + (2u * j[g] + go_right<NANP>(x[g], r[g].x, r[g].y)) * 4u);
+    for (int g = 0; g < G; ++g)
+      lf[g] = ld_sm<float>(base[g], kLeaf + (2u * j[g] + go_right<NANP>(x[g], r[g].x, r[g].y)) * 4u);
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       const float leaf = lf[g];
@@ -470,25 +482,25 @@ __device__ __forceinline__ float walk_chunk(uint32_t tb, int q, int nt, uint32_t
     }
   }
   for (; t < nt; t += Q) {
-    const uint32_t base = tb + static_cast<uint32_t>(t) * tree_bytes;
+    const unsigned char* base = tb + static_cast<uint32_t>(t) * tree_bytes;
     uint32_t j = 0;
 #pragma unroll
     for (int l = 0; l < D - 1; ++l) {
       uint32_t thr, meta;
       if (l < static_cast<int>(L.top)) {
-        const uint2 r = lds_u2(base + j * 8u);
+        const uint2 r = ld_sm<uint2>(base, j * 8u);
         thr = r.x;
         meta = r.y;
       } else {
-        meta = lds_u32(base + kMeta + j * 4u);
-        thr = lds_u32(base + kThr + j * 4u);
+        meta = ld_sm<uint32_t>(base, kMeta + j * 4u);
+        thr = ld_sm<uint32_t>(base, kThr + j * 4u);
       }
-      const float x = lds_f32(meta * row_bytes + xa);
+      const float x = ld_sm<float>(xc, meta * row_bytes);
       j = 2u * j + 1u + go_right<NANP>(x, thr, meta);
     }
-    const uint2 r = lds_u2(base + kLast + j * 8u);
-    const float x = lds_f32(r.y * row_bytes + xa);
-    const float leaf = lds_f32(base + kLeaf + (2u * j + go_right<NANP>(x, r.x, r.y)) * 4u);
+    const uint2 r = ld_sm<uint2>(base, kLast + j * 8u);
+    const float x = ld_sm<float>(xc, r.y * row_bytes);
+    const float leaf = ld_sm<float>(base, kLeaf + (2u * j + go_right<NANP>(x, r.x, r.y)) * 4u);
     if (Q == 1)
       acc += leaf;
     else
@@ -847,6 +859,7 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
   float acc = 0.0f;
   const uint32_t row_bytes = static_cast<uint32_t>(TC) * xb;
   const uint32_t xa = smem_u32(xs) + static_cast<uint32_t>(c) * xb;
+  const unsigned char* xcol = reinterpret_cast<const unsigned char*>(xs) + static_cast<uint32_t>(c) * xb;
   const uint32_t tbuf_a = smem_u32(tbuf);
   // parked leaves: buffer p holds leaf t of candidate c at la[p] + t * row_bytes
   const uint32_t la0 = smem_u32(smem + leaf_off) + static_cast<uint32_t>(c) * 4u;
@@ -877,8 +890,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
       else if constexpr (SH > 0)
         acc = walk_chunk_split<SH, G, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail, a.max_depth - SH);
       else
-        acc = nan ? walk_chunk<D, G, true, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u)
-                  : walk_chunk<D, G, false, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u);
+        acc = nan ? walk_chunk<D, G, true, 1>(tbuf + (tb - tbuf_a), 0, nt, a.tree_bytes, xcol, row_bytes, acc, 0u)
+                  : walk_chunk<D, G, false, 1>(tbuf + (tb - tbuf_a), 0, nt, a.tree_bytes, xcol, row_bytes, acc, 0u);
       __syncwarp();
       if (lane == 0 && ch + a.nbuf < n_chunks) {
         __threadfence_block();  // this warp's reads of buffer b are done
@@ -927,8 +940,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
     else if constexpr (SH > 0)
       acc = walk_chunk_split<SH, G, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail, a.max_depth - SH);
     else
-      acc = nan ? walk_chunk<D, G, true, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la)
-                : walk_chunk<D, G, false, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la);
+      acc = nan ? walk_chunk<D, G, true, Q>(tbuf + (tb - tbuf_a), q, nt, a.tree_bytes, xcol, row_bytes, acc, la)
+                : walk_chunk<D, G, false, Q>(tbuf + (tb - tbuf_a), q, nt, a.tree_bytes, xcol, row_bytes, acc, la);
     if (Q > 1 && q == 0 && ch > 0) {
       // the previous chunk's leaves (complete since the last barrier)
       const uint32_t lp = la0 + static_cast<uint32_t>((ch - 1) & 1) * la_step;
