@@ -395,8 +395,8 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  *                256 (<= 512 for split tables, 1,024 with 8 groups)
  *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10 and
  *                split tables), 4 or 8 (compact tables)
- *   chunk_trees  trees per shared-memory chunk, 1, 2, 4, 8 or 16 (full,
- *                half and split tables)
+ *   chunk_trees  trees per shared-memory chunk: 1, 2, 4, 8 or 16 (full,
+ *                half and split tables), 32 (split tables)
  *   nbuf         chunk buffers, 2 or 3 (full, half and split tables)
  * A shape that does not fit shared memory falls back to the library's
  * choice.  Results never depend on the shape.  Host-only. */

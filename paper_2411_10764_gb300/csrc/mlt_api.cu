@@ -1475,8 +1475,8 @@ int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk
     return fail(MLT_EINVAL, "splits must be 0, 1, 2, 4 or 8");
   if (!(group == 0 || group == 2 || group == 4 || group == 8)) return fail(MLT_EINVAL, "group must be 0, 2, 4 or 8");
   if (!(chunk_trees == 0 || chunk_trees == 1 || chunk_trees == 2 || chunk_trees == 4 || chunk_trees == 8 ||
-        chunk_trees == 16))
-    return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8 or 16");
+        chunk_trees == 16 || chunk_trees == 32))
+    return fail(MLT_EINVAL, "chunk_trees must be 0, 1, 2, 4, 8, 16 or 32");
   if (!(nbuf == 0 || nbuf == 2 || nbuf == 3)) return fail(MLT_EINVAL, "nbuf must be 0, 2 or 3");
   if (candidates && splits && candidates * splits > 1024)
     return fail(MLT_EINVAL, "candidates x splits must be at most 1024");

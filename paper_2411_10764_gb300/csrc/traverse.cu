@@ -146,7 +146,7 @@ ScreenShape plan_split(int F, int n_trees, uint32_t hb, long long n_eff, int sms
     for (int tc : {256, 128, 64, 32}) {
       if (ov.threads && tc != ov.threads) continue;
       if (tc * q > (q == 8 ? 1024 : 512)) continue;
-      for (int ch : {16, 8, 4}) {
+      for (int ch : {32, 16, 8, 4}) {
         if (ov.chunk_trees && ch != ov.chunk_trees) continue;
         const int chunk = std::min(ch, n_trees);
         for (int nb : {2, 3}) {

@@ -89,7 +89,8 @@ SPLIT_TABLE_SHAPES = ([(6, c, q, g, 8, 2) for c in (32, 64, 128) for q in (1, 2,
                       [(6, 64, 2, 4, ch, nb) for ch in (4, 16) for nb in (2, 3)] +
                       [(7, c, q, g, ch, 2) for c, q, g, ch in ((128, 4, 4, 16), (64, 2, 8, 16), (32, 1, 4, 4),
                                                                (128, 1, 8, 8), (128, 8, 2, 16), (32, 8, 2, 16))] +
-                      [(6, 64, 8, 4, 16, 3), (6, 128, 8, 2, 8, 2), (7, 128, 4, 2, 8, 3)])
+                      [(6, 64, 8, 4, 16, 3), (6, 128, 8, 2, 8, 2), (7, 128, 4, 2, 8, 3), (6, 128, 8, 4, 32, 2),
+                       (6, 64, 8, 2, 32, 2), (7, 128, 4, 2, 32, 2)])
 
 
 @pytest.mark.parametrize("head,cand,groups,group,chunk,nbuf", SPLIT_TABLE_SHAPES)
