@@ -402,6 +402,14 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  * choice.  Results never depend on the shape.  Host-only. */
 int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf);
 
+/* Tuning: batches of up to max_n candidates (0 .. 8,192; the default is
+ * 8,192) with stored features, whose V and P are full tables (depth <= 10)
+ * of the same depth small enough to share a CTA's shared memory, are
+ * screened by one kernel launch (V walk, validity, P walk, keys and the
+ * top-k selection by its last CTA) instead of four; 0 turns that path off.
+ * Results never depend on the path.  Host-only. */
+int mlt_tune_fused_small(int max_n);
+
 /* Tuning: the table format of models V and P deeper than 10 levels, for
  * ensembles loaded after this call.  levels = 6 (the default) or 7: a
  * split table, whose first `levels` levels stream through shared memory

@@ -134,6 +134,7 @@ ShapeOverride g_shape[3];
 // full-table V pass makes CTA g_stall_cta wait on a barrier phase that
 // nothing completes, for g_stall_ns (one shot)
 int g_head_levels = kSplitHeadDefault;  // split tables for deep V and P models (0: compact tables)
+long long g_small_max = kSmallMaxN;     // batches up to this size screen in one launch when eligible
 int g_stall_cta = -1;
 unsigned long long g_stall_ns = 0;
 
@@ -510,6 +511,27 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
     ev = &g_events[g_events_used];
     g_events_used += kPhases + 1;
     MLT_CUDA(cudaEventRecord(ev[0], st), "cudaEventRecord");
+  }
+  // a small batch of stored features: the whole step in one launch (its
+  // time is recorded as the V phase)
+  if (dec == nullptr && n <= g_small_max) {
+    const SmallPlan pl = plan_small(g_F, n, V, P, sm_count(), smem_optin());
+    if (pl.threads > 0) {
+      int stall = -1;
+      unsigned long long stall_ns = 0;
+      if (g_stall_cta >= 0) {
+        stall = static_cast<int>(std::min<long long>(g_stall_cta, pl.ctas - 1));
+        stall_ns = g_stall_ns;
+        g_stall_cta = -1;
+      }
+      MLT_CUDA(launch_screen_small(pl, V, P, feats, g_F, n, a.tau, out_pvalid, out_perf, out_topk, k, s, stall,
+                                   stall_ns, st),
+               "small-batch screening launch");
+      if (ev)
+        for (int i = 1; i <= kPhases; ++i) MLT_CUDA(cudaEventRecord(ev[i], st), "cudaEventRecord");
+      g_launches += 1;
+      return MLT_OK;
+    }
   }
   const long long tiles_v = (n + sv.threads - 1) / sv.threads;
   if (g_stall_cta >= 0 && V.kind != kTableCompact && tiles_v > 0) {
@@ -938,6 +960,13 @@ int mlt_load_ensemble(int model_id, const mlt_node* nodes, int n_trees, int dept
                  : pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
   if (rc != MLT_OK) return rc;
   return install_model(model_id, packed, dm);
+}
+
+int mlt_tune_fused_small(int max_n) {
+  if (max_n < 0 || max_n > kSmallMaxN) return fail(MLT_EINVAL, "max_n must lie in [0, %d], got %d", kSmallMaxN, max_n);
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_small_max = max_n;
+  return MLT_OK;
 }
 
 int mlt_tune_head_levels(int levels) {

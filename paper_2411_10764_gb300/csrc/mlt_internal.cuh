@@ -363,6 +363,22 @@ cudaError_t launch_sa_accept(long long space, const int64_t* parent, const float
                              float temperature, int64_t* out_next, float* out_next_score,
                              int32_t* out_accepted, cudaStream_t st);
 
+// screen_small.cu: the whole screening step in one launch for small batches
+// (full V and P tables of the same depth held in shared memory together)
+constexpr int kSmallMaxN = 8192;                 // candidates (keys the last CTA sorts)
+constexpr size_t kSmallTableBytes = 160 * 1024;  // V + P tables
+struct SmallPlan {
+  int threads = 0;  // candidates per CTA (0: not eligible)
+  int groups = 0;   // tree groups (CTA = 256 threads)
+  size_t smem = 0;
+  int ctas = 0;
+};
+SmallPlan plan_small(int F, long long n, const DeviceModel& V, const DeviceModel& P, int sms, int device_smem_optin);
+cudaError_t launch_screen_small(const SmallPlan& pl, const DeviceModel& V, const DeviceModel& P, const float* feats,
+                                int F, long long n, float tau, float* out_pvalid, float* out_perf, int64_t* out_topk,
+                                int k, const Scratch& sc, int stall_cta, unsigned long long stall_ns,
+                                cudaStream_t st);
+
 // selftest.cu: a bounded wait that runs out (failure-detection self-test)
 cudaError_t launch_wait_selftest(unsigned* err, unsigned long long limit_ns, cudaStream_t st);
 

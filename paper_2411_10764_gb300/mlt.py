@@ -74,6 +74,7 @@ def lib(build_if_missing: bool = True):
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
             "mlt_tune_head_levels": [i32],
+            "mlt_tune_fused_small": [i32],
             "mlt_walk_peak": [P, i32, P, i64, i32, P, P],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
@@ -426,6 +427,12 @@ def tune_walk(model_id: int, candidates: int = 0, splits: int = 0, group: int = 
     """Fix (or with zeros, release) the tree walk's launch shape for one model."""
     _check(lib().mlt_tune_walk(int(model_id), int(candidates), int(splits), int(group), int(chunk_trees),
                                int(nbuf)))
+
+
+def tune_fused_small(max_n: int) -> None:
+    """Batches up to max_n candidates (0 .. 8192) screen in one launch when
+    their models allow it; 0 turns the single-launch path off."""
+    _check(lib().mlt_tune_fused_small(int(max_n)))
 
 
 def tune_head_levels(levels: int) -> None:
