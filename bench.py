@@ -768,9 +768,9 @@ def run_ours(args):
             per_config[str(wid)] = rec
             del bufs, wc
             torch.cuda.empty_cache()
-        if not args.no_next:
-            extra = next_rows(ctx, W.make_workload(2, seed=seed), seed, args)
-            torch.cuda.empty_cache()
+    if world == 1 and not args.no_next:
+        extra = next_rows(ctx, W.make_workload(2, seed=seed), seed, args)
+        torch.cuda.empty_cache()
 
     if rank != 0:
         if dist is not None:
@@ -816,7 +816,7 @@ def main():
                     help="oracle time for each other workload's CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-config", action="store_true",
-                    help="only the headline workload (no per-workload records or next-row timings)")
+                    help="only the headline workload (no per-workload records)")
     ap.add_argument("--no-next", action="store_true",
                     help="skip the rerank, half-table, accumulation, explorer-step and decoder timings")
     ap.add_argument("--no-rerank", action="store_true", help=argparse.SUPPRESS)  # older command lines:
