@@ -386,13 +386,16 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
 
 /* Tuning: fix the launch shape of the tree walk over model `model_id`'s
  * trees (0 in any field = let the library choose it):
- *   candidates   candidates per CTA: a multiple of 32, 32 .. 256
+ *   candidates   candidates per CTA: a multiple of 32, 32 .. 384 (above
+ *                256 only for fp32 tables of depth <= 10 walked by one
+ *                group of warps; 32 .. 256 otherwise)
  *   splits       threads sharing one candidate's trees: 1, 2 or 4 for
  *                ensembles of depth <= 10, 1, 2, 4 or 8 for split tables
  *                (groups of warps, leaves summed in tree order through
  *                shared memory), 1, 2, 4 or 8 for compact tables (lanes of
  *                a warp, summed through shuffles); candidates x splits <=
- *                256 (<= 512 for split tables, 1,024 with 8 groups)
+ *                256 (384 with splits 1 for fp32 tables of depth <= 10,
+ *                512 for split tables, 1,024 with 8 groups)
  *   group        trees a thread walks at once: 2, 4 or 8 (depth <= 10 and
  *                split tables), 4 or 8 (compact tables)
  *   chunk_trees  trees per shared-memory chunk: 1, 2, 4, 8 or 16 (full,

@@ -398,19 +398,18 @@ int pack_ensemble(const mlt_node* nodes, int n_trees, int depth, int F, std::vec
         if (j < lay.n_top) {
           std::memcpy(dst + 8 * j, &thr_of[j], 4);
           std::memcpy(dst + 8 * j + 4, &meta_of[j], 4);
-        } else if (j < lay.n_inner) {
-          std::memcpy(dst + lay.off_thr + 4 * (j - lay.n_top), &thr_of[j], 4);
-          std::memcpy(dst + lay.off_meta + 4 * (j - lay.n_top), &meta_of[j], 4);
         } else {
-          const uint32_t q = j - lay.n_inner;
-          unsigned char* rec = dst + lay.off_last + 8 * q;
-          unsigned char* lv = dst + lay.off_last + 8 * (1u << (depth - 1)) + 8 * q;  // leaf pair
-          const float left = inherit[2 * j + 1], right = inherit[2 * j + 2];
-          std::memcpy(rec, &thr_of[j], 4);
-          std::memcpy(rec + 4, &meta_of[j], 4);
-          std::memcpy(lv, &left, 4);
-          std::memcpy(lv + 4, &right, 4);
+          // feature (< kMaxF) in bits 0..14, the NaN-left flag in bit 15
+          const uint16_t m = static_cast<uint16_t>((meta_of[j] & kMeta16Feature) |
+                                                   ((meta_of[j] & kMetaDefaultLeft) ? kMeta16Left : 0u));
+          std::memcpy(dst + lay.off_thr + 4 * (j - lay.n_top), &thr_of[j], 4);
+          std::memcpy(dst + lay.off_meta + 2 * (j - lay.n_top), &m, 2);
         }
+      }
+      // the leaf below each path: child heap index c of a last-level node
+      for (uint32_t c = static_cast<uint32_t>(inner); c < static_cast<uint32_t>(slots); ++c) {
+        const float v = inherit[c];
+        std::memcpy(dst + lay.off_leaf + 4 * (c - inner), &v, 4);
       }
     }
   } else {
@@ -1465,7 +1464,7 @@ int mlt_walk_peak(void* stream, int model_id, const float* feats, int64_t n, int
   const ScreenShape s = plan_for(dm, g_F, n, g_shape[model_id], true);
   if (s.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
   // one thread per candidate (a tree-group shape becomes one wider group)
-  const int tc = std::min(256, s.threads * s.lanes);
+  const int tc = std::min(kFullMaxTile, s.threads * s.lanes);
   const size_t feat_bytes = walk_peak_tree_offset(g_F, tc);
   int resident = std::min(dm.n_trees, s.chunk_trees * s.nbuf);
   while (resident > 1 && feat_bytes + static_cast<size_t>(resident) * dm.tree_bytes + 1024 > static_cast<size_t>(smem_optin()))
@@ -1498,8 +1497,8 @@ int mlt_walk_peak(void* stream, int model_id, const float* feats, int64_t n, int
 
 int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf) {
   if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
-  if (candidates < 0 || candidates > 256 || candidates % 32 != 0)
-    return fail(MLT_EINVAL, "candidates must be 0 or a multiple of 32 up to 256");
+  if (candidates < 0 || candidates > kFullMaxTile || candidates % 32 != 0)
+    return fail(MLT_EINVAL, "candidates must be 0 or a multiple of 32 up to %d", kFullMaxTile);
   if (!(splits == 0 || splits == 1 || splits == 2 || splits == 4 || splits == 8))
     return fail(MLT_EINVAL, "splits must be 0, 1, 2, 4 or 8");
   if (!(group == 0 || group == 2 || group == 4 || group == 8)) return fail(MLT_EINVAL, "group must be 0, 2, 4 or 8");

@@ -15,6 +15,7 @@ constexpr int kMaxProgram = 256;
 constexpr int kMaxF = 1024;
 constexpr int kMaxK = 16384;
 constexpr int kMaxDepth = 14;  // model A of the paper has depth 14 (Table 3)
+constexpr int kFullMaxTile = 384;  // candidates of a full-table tile walked by one group of warps
 constexpr int kMaxFullDepth = 10;  // deeper ensembles use the compact table
 
 // Device error bits (accumulated in one word, read by mlt_sync_status).
@@ -30,18 +31,18 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 // ---------------------------------------------------------------------------
 // Full table (depth D <= kMaxFullDepth): every tree is stored as a complete
 // binary tree of depth D, `tree_bytes` apart (a multiple of 16).  A node has
-// a threshold (float) and a meta word (bits 0..30 feature index, bit 31 NaN
-// goes left); its heap index is j (children 2j+1, 2j+2).  Each level is laid
-// out for the way a warp reads it (FullLayout below):
-//   levels [0, top)      : 8-byte records {threshold, meta} -- few distinct
-//                          nodes, mostly broadcast reads;
-//   levels [top, D-1)    : thresholds and metas in two 4-byte arrays -- a
-//                          32-lane gather of 4-byte words;
-//   level D-1 (last)     : 8-byte records {threshold, meta}, then the 2^D
-//                          leaves (leaf pair of last-level node q at 2q):
-//                          only the chosen leaf is read, which costs fewer
-//                          shared-memory wavefronts than one 16-byte record
-//                          holding both.
+// a threshold (float), a feature index (< kMaxF) and a NaN-goes-left flag;
+// its heap index is j (children 2j+1, 2j+2).  Each level is laid out for the
+// way a warp reads it (FullLayout below):
+//   levels [0, top)  : 8-byte records {threshold, meta} with meta = feature
+//                      | flag << 31 -- few distinct nodes, mostly broadcast
+//                      reads;
+//   levels [top, D)  : the thresholds as a 4-byte array and the metas as a
+//                      2-byte array (feature | flag << 15) -- 32-lane
+//                      gathers; 6 bytes a node where 8-byte records would
+//                      take 8, so more candidates and trees fit in shared
+//                      memory at once;
+//   then the 2^D leaves (4 bytes each, leaf i = child heap index - (2^D - 1)).
 // A shallower leaf is replicated into every leaf slot below it (its
 // pass-through nodes test feature 0; any path gives the leaf).
 //
@@ -106,26 +107,28 @@ constexpr uint32_t kHalfFeatureShift = 16;
 constexpr uint32_t kHalfFeatureMask = 0x3FFu;
 
 struct FullLayout {
-  uint32_t top;        // levels held as 8-byte records
-  uint32_t n_top;      // nodes in levels [0, top)
-  uint32_t n_inner;    // nodes in levels [0, D-1)
-  uint32_t off_thr;    // byte offset of the middle-level thresholds
-  uint32_t off_meta;   // byte offset of the middle-level metas
-  uint32_t off_last;   // byte offset of the last-level 8-byte records (the leaves follow them)
-  uint32_t bytes;      // bytes per tree (multiple of 16)
+  uint32_t top;       // levels held as 8-byte records
+  uint32_t n_top;     // nodes in levels [0, top)
+  uint32_t n_inner;   // nodes in levels [0, D)
+  uint32_t off_thr;   // byte offset of the thresholds of levels [top, D)
+  uint32_t off_meta;  // byte offset of their 2-byte metas
+  uint32_t off_leaf;  // byte offset of the 2^D leaves
+  uint32_t bytes;     // bytes per tree (multiple of 16)
 };
 
 __host__ __device__ constexpr FullLayout full_layout(int D) {
   const uint32_t top = D - 1 < 4 ? static_cast<uint32_t>(D - 1) : 4u;
   const uint32_t n_top = (1u << top) - 1u;
-  const uint32_t n_inner = (1u << (D - 1)) - 1u;
+  const uint32_t n_inner = (1u << D) - 1u;
   const uint32_t off_thr = n_top * 8u;
   const uint32_t off_meta = off_thr + (n_inner - n_top) * 4u;
-  const uint32_t off_last = (off_meta + (n_inner - n_top) * 4u + 15u) & ~15u;
-  // last level: 2^(D-1) 8-byte {threshold, meta} records, then 2^D leaves
-  const uint32_t bytes = off_last + (1u << (D - 1)) * 16u;
-  return FullLayout{top, n_top, n_inner, off_thr, off_meta, off_last, bytes};
+  const uint32_t off_leaf = (off_meta + (n_inner - n_top) * 2u + 3u) & ~3u;
+  const uint32_t bytes = (off_leaf + (1u << D) * 4u + 15u) & ~15u;
+  return FullLayout{top, n_top, n_inner, off_thr, off_meta, off_leaf, bytes};
 }
+constexpr uint32_t kMeta16Feature = 0x7FFFu;  // 2-byte meta: feature index
+constexpr uint32_t kMeta16Left = 0x8000u;     // 2-byte meta: NaN goes left
+static_assert(kMaxF <= static_cast<int>(kMeta16Feature) + 1, "feature index must fit a 2-byte meta");
 
 constexpr uint32_t kMetaLeaf = 1u << 30;
 constexpr uint32_t kMetaDefaultLeft = 1u << 31;

@@ -13,7 +13,7 @@ namespace walk {
 // streaming, no barrier between chunks.  out[i] = the fp32 sum, in walk
 // order, of the rounds x resident leaves candidate i reaches.
 template <int D, int G>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(kFullMaxTile)
     k_walk_peak(const __grid_constant__ TraverseArgs a, int resident, int rounds, float* out) {
   extern __shared__ __align__(128) unsigned char smem[];
   const int TC = blockDim.x;

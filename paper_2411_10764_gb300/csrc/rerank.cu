@@ -31,23 +31,21 @@ __device__ __forceinline__ uint32_t go_right_nan(float x, uint32_t thr_bits, uin
 __device__ float leaf_full(const unsigned char* tree, int D, const float* x) {
   const FullLayout L = full_layout(D);
   uint32_t j = 0;
-  for (int l = 0; l < D - 1; ++l) {
+  for (int l = 0; l < D; ++l) {
     uint32_t thr, meta;
     if (l < static_cast<int>(L.top)) {
       const uint2 r = __ldg(reinterpret_cast<const uint2*>(tree) + j);
       thr = r.x;
       meta = r.y;
     } else {
-      meta = __ldg(reinterpret_cast<const uint32_t*>(tree + L.off_meta) + (j - L.n_top));
+      const uint32_t m = __ldg(reinterpret_cast<const unsigned short*>(tree + L.off_meta) + (j - L.n_top));
+      meta = (m & kMeta16Feature) | ((m & kMeta16Left) ? kMetaDefaultLeft : 0u);
       thr = __ldg(reinterpret_cast<const uint32_t*>(tree + L.off_thr) + (j - L.n_top));
     }
     const float xv = __ldg(x + (meta & ~kMetaDefaultLeft));
     j = 2u * j + 1u + go_right_nan(xv, thr, meta);
   }
-  const uint2 r = __ldg(reinterpret_cast<const uint2*>(tree + L.off_last) + (j - L.n_inner));
-  const float xv = __ldg(x + (r.y & ~kMetaDefaultLeft));
-  const float* lv = reinterpret_cast<const float*>(tree + L.off_last + 8u * (1u << (D - 1)));
-  return __ldg(lv + 2u * (j - L.n_inner) + go_right_nan(xv, r.x, r.y));
+  return __ldg(reinterpret_cast<const float*>(tree + L.off_leaf) + (j - L.n_inner));
 }
 
 // One tree of a compact table (breadth-first records).

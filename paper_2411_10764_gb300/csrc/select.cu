@@ -29,7 +29,7 @@ constexpr int kSortMin = 8192;  // collected keys held in shared memory
 constexpr unsigned kRankMax = 512;    // order by rank counting up to this many keys
 constexpr unsigned kDirectMax = 512;  // rank a collection this small without narrowing it
 
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(kFullMaxTile)
     k_scatter(const uint32_t* masks, const uint32_t* offsets, uint32_t* rows, long long n, const StreamState* ss) {
   __shared__ unsigned wc[32];
   pdl_wait();

@@ -43,7 +43,9 @@ FullKernelPtr full_kernel(int depth, int group, int q) {
 //   * a thread walks 8 trees at once (4 with tree groups when more than 8
 //     warps share the SM), the chunk permitting;
 //   * a batch of under 32 (64) candidates per SM splits each tile's trees
-//     over 4 (2) groups of warps.
+//     over 4 (2) groups of warps;
+//   * one CTA per SM whose chunks hold fewer than 8 trees grows past 256
+//     candidates, up to 384 (below).
 ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms, int optin,
                       const ShapeOverride& ov, bool half) {
   if (sms < 1) sms = 1;
@@ -77,7 +79,7 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
   } else {
     tc = ov.threads;
   }
-  if (tc * q > 256) return ScreenShape{};
+  if (tc * q > (q == 1 && !half ? kFullMaxTile : 256)) return ScreenShape{};
   const long long tiles = (n_eff + tc - 1) / tc;
   const long long tiles_sm = (tiles + sms - 1) / sms;
   ScreenShape best{};
@@ -112,6 +114,24 @@ ScreenShape plan_full(int F, int n_trees, uint32_t tb, long long n_eff, int sms,
         best.resident = std::max(1, res);
         best.sync_free = q == 1 && best.resident == 1 ? 1 : 0;
       }
+    }
+  }
+  // one CTA of 256 candidates per SM, no tree groups, fewer than 8 trees in
+  // flight per thread (large trees: the chunk holds few): the walk waits on
+  // its dependent shared-memory reads, so grow the tile (more warps) while
+  // the same chunks still fit and the busiest SM keeps two or more tiles.
+  // Measured on workload 4 (depth 10, 4-tree chunks, 96 decoded features):
+  // V pass 9.67 / 9.48 / 8.66 / 7.93 / 7.36 ms at 256 / 288 / 320 / 352 /
+  // 384 candidates.  With 8 trees in flight the shared-memory pipe is
+  // already busy, and a larger tile was slower (workload 3: 2.00 ms at 256
+  // candidates, 2.19 ms at 288).
+  if (best.threads == 256 && q == 1 && !half && best.resident == 1 && best.group < 8 && !ov.threads) {
+    for (int t2 = kFullMaxTile; t2 > 256; t2 -= 32) {
+      const size_t smem = smem_of(t2, best.chunk_trees, best.nbuf);
+      if (!fits(smem) || (n_eff + t2 - 1) / t2 < 2LL * sms) continue;
+      best.threads = t2;
+      best.smem = smem;
+      break;
     }
   }
   return best;  // threads == 0: nothing fits

@@ -410,8 +410,8 @@ __device__ __forceinline__ void sts_f32(uint32_t a, float v) {
 // xa = shared address of this thread's feature column (feature f at xa + f *
 // row_bytes).  Q == 1: the leaves are added to acc in tree order.  Q > 1:
 // leaf t is parked at la + t * row_bytes for an in-order sum afterwards.
-// The 32-bit product meta * row_bytes drops meta's bit 31 because row_bytes
-// is a multiple of 2.
+// The 32-bit product meta * row_bytes drops a 4-byte meta's bit 31 because
+// row_bytes is a multiple of 2; a 2-byte meta is masked to its feature.
 // Shared-memory loads of the walk as ordinary C++ loads through pointers
 // derived from the kernel's shared array (so they compile to shared-memory
 // loads the compiler may schedule freely among the G walks); the mbarrier
@@ -422,15 +422,39 @@ __device__ __forceinline__ T ld_sm(const unsigned char* p, uint32_t off) {
   return *reinterpret_cast<const T*>(p + off);
 }
 
+// Node j of a full-table tree at level l (a compile-time constant after
+// unrolling): threshold bits, the feature's byte offset in the staged tile,
+// and the NaN-goes-left flag in bit 31.
+template <int D>
+struct FullNode {
+  uint32_t thr, xoff, left;
+};
+template <int D>
+__device__ __forceinline__ FullNode<D> full_node(const unsigned char* base, int l, uint32_t j, uint32_t row_bytes) {
+  constexpr FullLayout L = full_layout(D);
+  // byte offsets folded with the heap index of each region's first node
+  constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
+  constexpr uint32_t kMeta = L.off_meta - L.n_top * 2u;
+  FullNode<D> n;
+  if (l < static_cast<int>(L.top)) {
+    const uint2 r = ld_sm<uint2>(base, j * 8u);
+    n.thr = r.x;
+    n.xoff = r.y * row_bytes;
+    n.left = r.y;
+  } else {
+    const uint32_t m = ld_sm<unsigned short>(base, kMeta + j * 2u);
+    n.thr = ld_sm<uint32_t>(base, kThr + j * 4u);
+    n.xoff = (m & kMeta16Feature) * row_bytes;
+    n.left = m << 16;
+  }
+  return n;
+}
+
 template <int D, int G, bool NANP, int Q>
 __device__ __forceinline__ float walk_chunk(const unsigned char* tb, int q, int nt, uint32_t tree_bytes,
                                             const unsigned char* xc, uint32_t row_bytes, float acc, uint32_t la) {
   constexpr FullLayout L = full_layout(D);
-  // byte offsets folded with the heap index of each region's first node
-  constexpr uint32_t kThr = L.off_thr - L.n_top * 4u;
-  constexpr uint32_t kMeta = L.off_meta - L.n_top * 4u;
-  constexpr uint32_t kLast = L.off_last - L.n_inner * 8u;
-  constexpr uint32_t kLeaf = L.off_last + (1u << (D - 1)) * 8u - L.n_inner * 8u;
+  constexpr uint32_t kLeaf = L.off_leaf - L.n_inner * 4u;  // leaf of child heap index c at kLeaf + 4c
   int t = q;
   for (; t + (G - 1) * Q < nt; t += G * Q) {
     const unsigned char* base[G];
@@ -441,66 +465,37 @@ __device__ __forceinline__ float walk_chunk(const unsigned char* tb, int q, int 
       j[g] = 0;
     }
 #pragma unroll
-    for (int l = 0; l < D - 1; ++l) {
-      uint32_t thr[G], meta[G];
-      if (l < static_cast<int>(L.top)) {
+    for (int l = 0; l < D; ++l) {
+      FullNode<D> n[G];
 #pragma unroll
-        for (int g = 0; g < G; ++g) {
-          const uint2 r = ld_sm<uint2>(base[g], j[g] * 8u);
-          thr[g] = r.x;
-          meta[g] = r.y;
-        }
-      } else {
-#pragma unroll
-        for (int g = 0; g < G; ++g) meta[g] = ld_sm<uint32_t>(base[g], kMeta + j[g] * 4u);
-#pragma unroll
-        for (int g = 0; g < G; ++g) thr[g] = ld_sm<uint32_t>(base[g], kThr + j[g] * 4u);
-      }
+      for (int g = 0; g < G; ++g) n[g] = full_node<D>(base[g], l, j[g], row_bytes);
       float x[G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, meta[g] * row_bytes);
+      for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, n[g].xoff);
 #pragma unroll
-      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], thr[g], meta[g]);
+      for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right<NANP>(x[g], n[g].thr, n[g].left);
     }
-    uint2 r[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) r[g] = ld_sm<uint2>(base[g], kLast + j[g] * 8u);
-    float x[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, r[g].y * row_bytes);
     float lf[G];
 #pragma unroll
-    for (int g = 0; g < G; ++g)
-      lf[g] = ld_sm<float>(base[g], kLeaf + (2u * j[g] + go_right<NANP>(x[g], r[g].x, r[g].y)) * 4u);
+    for (int g = 0; g < G; ++g) lf[g] = ld_sm<float>(base[g], kLeaf + j[g] * 4u);
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      const float leaf = lf[g];
       if (Q == 1)
-        acc += leaf;
+        acc += lf[g];
       else
-        sts_f32(la + static_cast<uint32_t>(t + g * Q) * row_bytes, leaf);
+        sts_f32(la + static_cast<uint32_t>(t + g * Q) * row_bytes, lf[g]);
     }
   }
   for (; t < nt; t += Q) {
     const unsigned char* base = tb + static_cast<uint32_t>(t) * tree_bytes;
     uint32_t j = 0;
 #pragma unroll
-    for (int l = 0; l < D - 1; ++l) {
-      uint32_t thr, meta;
-      if (l < static_cast<int>(L.top)) {
-        const uint2 r = ld_sm<uint2>(base, j * 8u);
-        thr = r.x;
-        meta = r.y;
-      } else {
-        meta = ld_sm<uint32_t>(base, kMeta + j * 4u);
-        thr = ld_sm<uint32_t>(base, kThr + j * 4u);
-      }
-      const float x = ld_sm<float>(xc, meta * row_bytes);
-      j = 2u * j + 1u + go_right<NANP>(x, thr, meta);
+    for (int l = 0; l < D; ++l) {
+      const FullNode<D> n = full_node<D>(base, l, j, row_bytes);
+      const float x = ld_sm<float>(xc, n.xoff);
+      j = 2u * j + 1u + go_right<NANP>(x, n.thr, n.left);
     }
-    const uint2 r = ld_sm<uint2>(base, kLast + j * 8u);
-    const float x = ld_sm<float>(xc, r.y * row_bytes);
-    const float leaf = ld_sm<float>(base, kLeaf + (2u * j + go_right<NANP>(x, r.x, r.y)) * 4u);
+    const float leaf = ld_sm<float>(base, kLeaf + j * 4u);
     if (Q == 1)
       acc += leaf;
     else
@@ -966,12 +961,12 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
 }
 
 template <int D, int G, int Q>
-__global__ void __launch_bounds__(256) k_traverse_full(const __grid_constant__ TraverseArgs a) {
+__global__ void __launch_bounds__(Q <= 1 ? kFullMaxTile : 256) k_traverse_full(const __grid_constant__ TraverseArgs a) {
   traverse_full_body<D, G, Q>(a, nullptr);
 }
 
 template <int D, int G, int Q>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(Q <= 1 ? kFullMaxTile : 256)
     k_traverse_full_dec(const __grid_constant__ TraverseArgs a, const __grid_constant__ DecodeParams d) {
   traverse_full_body<D, G, Q>(a, &d);
 }

@@ -133,7 +133,7 @@ def test_decoder_validation(L):
 
 @pytest.mark.parametrize("args", [(0, 48, 1, 4, 0, 0), (0, 64, 3, 4, 0, 0), (0, 256, 8, 4, 0, 0),
                                   (0, 64, 4, 3, 0, 0), (5, 64, 4, 4, 0, 0), (0, 0, 0, 0, 3, 0),
-                                  (0, 0, 0, 0, 0, 4), (0, 288, 1, 4, 0, 0)])
+                                  (0, 0, 0, 0, 0, 4), (0, 416, 1, 4, 0, 0)])
 def test_walk_tuning_rejects(args):
     with pytest.raises(mlt.MltError):
         mlt.tune_walk(*args)
@@ -142,7 +142,9 @@ def test_walk_tuning_rejects(args):
 def test_walk_tuning_accepts_and_releases():
     mlt.tune_walk(mlt.MLT_MODEL_P, 64, 4, 8, 8, 2)
     mlt.tune_walk(mlt.MLT_MODEL_P, 96, 2, 2, 16, 3)
+    mlt.tune_walk(mlt.MLT_MODEL_V, 384, 1, 4, 4, 2)
     mlt.tune_walk(mlt.MLT_MODEL_P)
+    mlt.tune_walk(mlt.MLT_MODEL_V)
 
 
 @pytest.mark.parametrize("case", ["model_a", "depth_11", "leaf_past_binary16", "invalid_tree"])

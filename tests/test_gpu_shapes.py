@@ -120,7 +120,8 @@ def test_split_walk_decoded_shapes(deep_decoded, head, cand, groups, group):
     assert_parity(got, _expected("deep_decoded", deep_decoded))
 
 
-FULL_SHAPES = [(t, c, b) for t in (32, 64, 128, 256) for c in (1, 2, 4, 8, 16) for b in (2, 3)]
+FULL_SHAPES = ([(t, c, b) for t in (32, 64, 128, 256) for c in (1, 2, 4, 8, 16) for b in (2, 3)] +
+               [(t, c, 2) for t in (288, 384) for c in (4, 16)])
 
 
 @pytest.mark.parametrize("threads,chunk,nbuf", FULL_SHAPES)
@@ -148,7 +149,7 @@ def test_full_walk_tree_groups(full, cand, splits, group, chunk):
     assert_parity(got, _expected("full", full))
 
 
-@pytest.mark.parametrize("cand", [96, 160, 224])
+@pytest.mark.parametrize("cand", [96, 160, 224, 320, 352])
 def test_full_walk_candidate_counts_not_powers_of_two(full, cand):
     try:
         _force(candidates=cand)
@@ -163,7 +164,8 @@ def decoded():
     return W.make_workload(4, seed=3, n=7001)
 
 
-@pytest.mark.parametrize("cand,splits,group,chunk", [(128, 2, 8, 16), (64, 4, 4, 8), (96, 2, 4, 4), (256, 1, 8, 4)])
+@pytest.mark.parametrize("cand,splits,group,chunk", [(128, 2, 8, 16), (64, 4, 4, 8), (96, 2, 4, 4), (256, 1, 8, 4),
+                                                     (352, 1, 4, 4), (384, 1, 2, 2)])
 def test_full_walk_decoded_shapes(decoded, cand, splits, group, chunk):
     try:
         _force(candidates=cand, splits=splits, group=group, chunk_trees=chunk, nbuf=2)
