@@ -658,13 +658,23 @@ __device__ __forceinline__ uint32_t go_right_split(float x, uint32_t thr_bits, u
   return !(xs < __uint_as_float(thr_bits)) ? 1u : 0u;
 }
 
+// A tail record load that only the live walkers issue (v keeps its value
+// where p is false), so the tail loop has no branch per walker.
+__device__ __forceinline__ void ldg_u2_hint_if(bool p, const uint2* ptr, unsigned long long pol, uint2& v) {
+  asm("{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %3, 0;\n\t"
+      "@q ld.global.nc.L2::cache_hint.v2.u32 {%0, %1}, [%2], %4;\n\t}"
+      : "+r"(v.x), "+r"(v.y)
+      : "l"(ptr), "r"(p ? 1 : 0), "l"(pol));
+}
+
 template <int H, int G, int Q>
-__device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, uint32_t head_bytes, uint32_t xa,
-                                                  uint32_t row_bytes, float acc, uint32_t la, const uint2* tails,
-                                                  int tail_steps) {
+__device__ __forceinline__ float walk_chunk_split(const unsigned char* tb, int q, int nt, uint32_t head_bytes,
+                                                  const unsigned char* xc, uint32_t row_bytes, float acc, uint32_t la,
+                                                  const uint2* tails, int tail_steps) {
   const unsigned long long keep = policy_evict_last();
   for (int t = q; t < nt; t += G * Q) {
-    uint32_t base[G], j[G];
+    const unsigned char* base[G];
+    uint32_t j[G];
     bool in[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
@@ -676,10 +686,10 @@ __device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, ui
     for (int l = 0; l < H; ++l) {
       uint2 r[G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) r[g] = lds_u2(base[g] + j[g] * 8u);
+      for (int g = 0; g < G; ++g) r[g] = ld_sm<uint2>(base[g], j[g] * 8u);
       float x[G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) x[g] = lds_f32(r[g].y * row_bytes + xa);
+      for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, r[g].y * row_bytes);
 #pragma unroll
       for (int g = 0; g < G; ++g) j[g] = 2u * j[g] + 1u + go_right_split(x[g], r[g].x, r[g].y);
     }
@@ -689,26 +699,25 @@ __device__ __forceinline__ float walk_chunk_split(uint32_t tb, int q, int nt, ui
     bool live[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      r[g] = lds_u2(base[g] + j[g] * 8u);
-      tbase[g] = lds_u32(base[g] + head_bytes - 8u);
+      r[g] = ld_sm<uint2>(base[g], j[g] * 8u);
+      tbase[g] = ld_sm<uint32_t>(base[g], head_bytes - 8u);
       live[g] = in[g] && !(r[g].y & kMetaLeaf);
     }
     bool any = false;
 #pragma unroll
     for (int g = 0; g < G; ++g) any |= live[g];
+    // every walker computes its next index (a leaf record reads feature 0
+    // and child 0); only the live ones load
     for (int s = 0; s < tail_steps && __any_sync(0xFFFFFFFFu, any); ++s) {
-      uint32_t idx[G];
+      float x[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) x[g] = ld_sm<float>(xc, (r[g].y & kCompactFeatureMask) * row_bytes);
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        idx[g] = 0;
-        if (live[g]) {
-          const float x = lds_f32((r[g].y & kCompactFeatureMask) * row_bytes + xa);
-          idx[g] = tbase[g] + ((r[g].y >> kCompactChildShift) & kCompactChildMask) + go_right_split(x, r[g].x, r[g].y);
-        }
+        const uint32_t idx =
+            tbase[g] + ((r[g].y >> kCompactChildShift) & kCompactChildMask) + go_right_split(x[g], r[g].x, r[g].y);
+        ldg_u2_hint_if(live[g], tails + idx, keep, r[g]);
       }
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-        if (live[g]) r[g] = ldg_u2_hint(tails + idx[g], keep);
       any = false;
 #pragma unroll
       for (int g = 0; g < G; ++g) {
@@ -883,7 +892,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
         acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                   : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
       else if constexpr (SH > 0)
-        acc = walk_chunk_split<SH, G, 1>(tb, 0, nt, a.tree_bytes, xa, row_bytes, acc, 0u, a.tail, a.max_depth - SH);
+        acc = walk_chunk_split<SH, G, 1>(tbuf + (tb - tbuf_a), 0, nt, a.tree_bytes, xcol, row_bytes, acc, 0u, a.tail,
+                                         a.max_depth - SH);
       else
         acc = nan ? walk_chunk<D, G, true, 1>(tbuf + (tb - tbuf_a), 0, nt, a.tree_bytes, xcol, row_bytes, acc, 0u)
                   : walk_chunk<D, G, false, 1>(tbuf + (tb - tbuf_a), 0, nt, a.tree_bytes, xcol, row_bytes, acc, 0u);
@@ -933,7 +943,8 @@ __device__ __forceinline__ void traverse_full_body(const TraverseArgs& a, const 
       acc = nan ? walk_chunk_half<D, G, true>(tb, nt, a.tree_bytes, xa, row_bytes, acc)
                 : walk_chunk_half<D, G, false>(tb, nt, a.tree_bytes, xa, row_bytes, acc);
     else if constexpr (SH > 0)
-      acc = walk_chunk_split<SH, G, Q>(tb, q, nt, a.tree_bytes, xa, row_bytes, acc, la, a.tail, a.max_depth - SH);
+      acc = walk_chunk_split<SH, G, Q>(tbuf + (tb - tbuf_a), q, nt, a.tree_bytes, xcol, row_bytes, acc, la, a.tail,
+                                       a.max_depth - SH);
     else
       acc = nan ? walk_chunk<D, G, true, Q>(tbuf + (tb - tbuf_a), q, nt, a.tree_bytes, xcol, row_bytes, acc, la)
                 : walk_chunk<D, G, false, Q>(tbuf + (tb - tbuf_a), q, nt, a.tree_bytes, xcol, row_bytes, acc, la);
