@@ -14,10 +14,10 @@
 //   * group 0 decides validity against tau, writes pvalid and perf, and
 //     appends a rank key per valid candidate;
 //   * the last CTA to finish (a ticket, no waiting) selects the top-k: a
-//     12-bit histogram of the keys in shared memory gives the bucket of the
-//     k-th key, the keys at or above it are ranked directly (each counts the
-//     larger ones), and a bitonic sort of all keys serves when that bucket
-//     holds too many.
+//     histogram of the keys over equal-width bins of the batch's score range
+//     gives the bin of the k-th key, the keys at or above it are ranked
+//     directly (each counts the larger ones), and a bitonic sort of all keys
+//     serves when that bin holds too many.
 #include <algorithm>
 
 #include "rank.cuh"
@@ -30,7 +30,7 @@ using namespace walk;
 
 constexpr int kSmallThreads = 256;
 constexpr int kSmallSortMax = kSmallMaxN;  // keys the last CTA can sort (a power of two)
-constexpr int kSmallHistBins = 4096;       // top 12 bits of a key
+constexpr int kSmallHistBins = 1024;       // equal-width bins over the batch's score range
 constexpr unsigned kSmallRankMax = 512;    // rank a collection this small directly
 
 struct SmallArgs {
@@ -67,35 +67,80 @@ __host__ __device__ constexpr size_t small_select_bytes() {
   return (static_cast<size_t>(kSmallSortMax) + 2) * 8 + kSmallHistBins * 4 + (kSmallRankMax + 2) * 8;
 }
 
-// The top-k of the keys[0, m) (m <= kSmallSortMax) by the last CTA.
+// The top-k of the keys[0, m) (m <= kSmallSortMax) by the last CTA.  The
+// keys come in with every load of a thread in flight at once.  Up to
+// kSmallRankMax keys are ranked directly.  Otherwise a histogram over
+// equal-width bins of the score words' range [lo, hi] (bin = (score - lo) x
+// scale, non-decreasing in the key, so a better key never lands in a lower
+// bin) gives the bin of the kk-th key; the keys in that bin and above are
+// collected and ranked, or, if that bin holds too many (equal scores), every
+// key is sorted.  Equal-width bins spread a batch's scores over the
+// histogram where the top bits of the keys put them in a handful of bins.
+__device__ __forceinline__ unsigned small_bin(unsigned long long key, unsigned lo, float scale) {
+  const unsigned b = static_cast<unsigned>(static_cast<float>(static_cast<unsigned>(key >> 32) - lo) * scale);
+  return b < static_cast<unsigned>(kSmallHistBins) ? b : static_cast<unsigned>(kSmallHistBins) - 1u;
+}
+
 __device__ __forceinline__ void select_small(const SmallArgs& s, unsigned m, unsigned char* smem) {
+  constexpr int kUnroll = 8;
   const int T = blockDim.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  __shared__ unsigned warp_sum[kSmallThreads / 32];
-  __shared__ unsigned s_bin, s_cnt;
+  __shared__ unsigned warp_sum[kSmallThreads / 32], warp_lo[kSmallThreads / 32], warp_hi[kSmallThreads / 32];
+  __shared__ unsigned s_bin;
   unsigned long long* ks = reinterpret_cast<unsigned long long*>(smem);
   unsigned* hist = reinterpret_cast<unsigned*>(ks + kSmallSortMax + 2);
   unsigned long long* cs = reinterpret_cast<unsigned long long*>(hist + kSmallHistBins);
   const unsigned kk = m < static_cast<unsigned>(s.k) ? m : static_cast<unsigned>(s.k);
-  for (unsigned i = tid; i < m; i += T) ks[i] = __ldcg(s.keys + i);
+  unsigned lo = 0xFFFFFFFFu, hi = 0u;
+  for (unsigned i0 = 0; i0 < m; i0 += static_cast<unsigned>(T) * kUnroll) {
+    unsigned long long v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const unsigned i = i0 + static_cast<unsigned>(u * T + tid);
+      v[u] = i < m ? __ldcg(s.keys + i) : 0ull;
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const unsigned i = i0 + static_cast<unsigned>(u * T + tid);
+      if (i < m) {
+        ks[i] = v[u];
+        const unsigned w = static_cast<unsigned>(v[u] >> 32);
+        lo = min(lo, w);
+        hi = max(hi, w);
+      }
+    }
+  }
   if (kk > 0) {
     if (m <= kSmallRankMax) {
       if (tid == 0 && (m & 1u)) ks[m] = 0ull;
       __syncthreads();
       rank_and_write(ks, m, kk, 0, s.out_topk);
     } else {
-      for (int b = tid; b < kSmallHistBins; b += T) hist[b] = 0u;
-      if (tid == 0) {
-        s_bin = 0u;
-        s_cnt = 0u;
+      lo = __reduce_min_sync(0xFFFFFFFFu, lo);
+      hi = __reduce_max_sync(0xFFFFFFFFu, hi);
+      if (lane == 0) {
+        warp_lo[warp] = lo;
+        warp_hi[warp] = hi;
       }
+      for (int b = tid; b < kSmallHistBins; b += T) hist[b] = 0u;
+      if (tid == 0) s_bin = 0u;
       __syncthreads();
-      for (unsigned i = tid; i < m; i += T) atomicAdd(&hist[ks[i] >> (64 - 12)], 1u);
+      for (int w = 0; w < T / 32; ++w) {
+        lo = min(lo, warp_lo[w]);
+        hi = max(hi, warp_hi[w]);
+      }
+      const float scale = hi > lo ? (static_cast<float>(kSmallHistBins) - 0.5f) / static_cast<float>(hi - lo) : 0.0f;
+      for (unsigned i = tid; i < m; i += T) atomicAdd(&hist[small_bin(ks[i], lo, scale)], 1u);
       __syncthreads();
-      // bucket of the kk-th largest key: thread t holds the 16 bins just
-      // below 4096 - 16 t, threads ordered from the top bins down
+      // bin of the kk-th largest key: thread t holds the `per` bins just
+      // below kSmallHistBins - per t, threads ordered from the top bins down
       constexpr int per = kSmallHistBins / kSmallThreads;
+      unsigned h[per];
       unsigned local = 0;
-      for (int b = 0; b < per; ++b) local += hist[kSmallHistBins - 1 - (tid * per + b)];
+#pragma unroll
+      for (int b = 0; b < per; ++b) {
+        h[b] = hist[kSmallHistBins - 1 - (tid * per + b)];
+        local += h[b];
+      }
       unsigned x = local;
       for (int o = 1; o < 32; o <<= 1) {
         const unsigned y = __shfl_up_sync(0xFFFFFFFFu, x, o);
@@ -105,30 +150,44 @@ __device__ __forceinline__ void select_small(const SmallArgs& s, unsigned m, uns
       __syncthreads();
       unsigned above = x - local;
       for (int w = 0; w < warp; ++w) above += warp_sum[w];
+#pragma unroll
       for (int b = 0; b < per; ++b) {
-        const unsigned bin = kSmallHistBins - 1 - (tid * per + b);
-        const unsigned h = hist[bin];
-        if (above < kk && kk <= above + h) s_bin = bin;
-        above += h;
+        if (above < kk && kk <= above + h[b]) s_bin = static_cast<unsigned>(kSmallHistBins - 1 - (tid * per + b));
+        above += h[b];
       }
       __syncthreads();
-      // the keys of that bucket and above (every key better than the kk-th)
-      const unsigned long long bin = s_bin;
-      for (unsigned i = tid; i < m; i += T) {
-        const unsigned long long key = ks[i];
-        if ((key >> (64 - 12)) >= bin) {
-          const unsigned p = atomicAdd(&s_cnt, 1u);
-          if (p < kSmallRankMax) cs[p] = key;
+      // the keys of that bin and above (every key better than the kk-th):
+      // each thread counts its own, a block scan places them
+      const unsigned bin0 = s_bin;
+      unsigned mine = 0;
+      for (unsigned i = tid; i < m; i += T) mine += small_bin(ks[i], lo, scale) >= bin0 ? 1u : 0u;
+      unsigned xs = mine;
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned y = __shfl_up_sync(0xFFFFFFFFu, xs, o);
+        if (lane >= o) xs += y;
+      }
+      if (lane == 31) warp_sum[warp] = xs;
+      __syncthreads();
+      unsigned pos = xs - mine, cnt = 0;
+      for (int w = 0; w < T / 32; ++w) {
+        if (w < warp) pos += warp_sum[w];
+        cnt += warp_sum[w];
+      }
+      if (mine)
+        for (unsigned i = tid; i < m; i += T) {
+          const unsigned long long key = ks[i];
+          if (small_bin(key, lo, scale) >= bin0) {
+            if (pos < kSmallRankMax) cs[pos] = key;
+            ++pos;
+          }
         }
-      }
       __syncthreads();
-      const unsigned cnt = s_cnt;
       if (cnt <= kSmallRankMax) {
         if (tid == 0 && (cnt & 1u)) cs[cnt] = 0ull;
         __syncthreads();
         rank_and_write(cs, cnt, kk, 0, s.out_topk);
       } else {
-        // a crowded bucket: order every key
+        // a crowded bin: order every key
         int n2 = 2;
         while (n2 < static_cast<int>(m)) n2 <<= 1;
         for (int i = static_cast<int>(m) + tid; i < n2; i += T) ks[i] = 0ull;
@@ -145,7 +204,8 @@ __device__ __forceinline__ void select_small(const SmallArgs& s, unsigned m, uns
 template <int D, int G, int Q>
 __global__ void __launch_bounds__(kSmallThreads) k_screen_small(const __grid_constant__ SmallArgs s) {
   extern __shared__ __align__(128) unsigned char smem[];
-  __shared__ __align__(8) unsigned long long bars[2];  // [1]: the self-test's stalled barrier
+  // [0] V table, [2] P table, [1] the self-test's stalled barrier
+  __shared__ __align__(8) unsigned long long bars[3];
   __shared__ unsigned s_last;
   const int TC = blockDim.x / Q;
   const int tid = threadIdx.x;
@@ -160,16 +220,16 @@ __global__ void __launch_bounds__(kSmallThreads) k_screen_small(const __grid_con
   float* park = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(xs) + align128(static_cast<size_t>(s.F) * TC * 4));
   const bool stall = static_cast<int>(blockIdx.x) == s.stall_cta;
   if (tid == 0) {
-    mbar_init(smem_u32(&bars[0]), 1);
-    mbar_init(smem_u32(&bars[1]), 1);
+    for (int b = 0; b < 3; ++b) mbar_init(smem_u32(&bars[b]), 1);
     fence_mbar_init();
   }
   __syncthreads();
   if (tid == 0) {  // the tables are static: copy them before waiting on earlier kernels
-    const uint32_t bar = smem_u32(&bars[0]);
-    mbar_expect_tx(bar, static_cast<uint32_t>(v_bytes + p_bytes));
-    bulk_copy_g2s(smem_u32(vt), s.v_table, static_cast<uint32_t>(v_bytes), bar);
-    bulk_copy_g2s(smem_u32(pt), s.p_table, static_cast<uint32_t>(p_bytes), bar);
+    // separate barriers, so that the V walk starts while the P table lands
+    mbar_expect_tx(smem_u32(&bars[0]), static_cast<uint32_t>(v_bytes));
+    bulk_copy_g2s(smem_u32(vt), s.v_table, static_cast<uint32_t>(v_bytes), smem_u32(&bars[0]));
+    mbar_expect_tx(smem_u32(&bars[2]), static_cast<uint32_t>(p_bytes));
+    bulk_copy_g2s(smem_u32(pt), s.p_table, static_cast<uint32_t>(p_bytes), smem_u32(&bars[2]));
   }
   pdl_wait();
   TraverseArgs ta{};
@@ -179,15 +239,9 @@ __global__ void __launch_bounds__(kSmallThreads) k_screen_small(const __grid_con
   const bool nan = __syncthreads_or(tid < TC && stage_row(ta, nullptr, xs, nullptr, tile0, rows_here, TC));
   const bool ok = stall ? mbar_wait_bounded_ns(smem_u32(&bars[1]), 0u, s.stall_ns)
                         : mbar_wait_bounded(smem_u32(&bars[0]), 0u);
-  const bool failed = !__syncthreads_and(ok);
+  bool failed = !__syncthreads_and(ok);
   float accv = 0.0f, accp = 0.0f;
-  if (failed) {
-    if (tid == 0) {
-      mbar_wait_bounded(smem_u32(&bars[0]), 0u);  // the copies land before the CTA's shared memory is released
-      atomicOr(s.err, kErrWaitTimeout);
-    }
-    accv = -INFINITY;  // the tile's bookkeeping still completes, none of it valid
-  } else {
+  if (!failed) {
     const uint32_t row_bytes = static_cast<uint32_t>(TC) * 4u;
     const unsigned char* xcol = reinterpret_cast<const unsigned char*>(xs) + static_cast<uint32_t>(c) * 4u;
     const uint32_t la = smem_u32(park) + static_cast<uint32_t>(c) * 4u;
@@ -199,13 +253,25 @@ __global__ void __launch_bounds__(kSmallThreads) k_screen_small(const __grid_con
         for (int t = 0; t < s.v_trees; ++t) accv += park[t * TC + c];
       __syncthreads();
     }
-    accp = nan ? walk_chunk<D, G, true, Q>(pt, q, s.p_trees, s.tree_bytes, xcol, row_bytes, 0.0f, la)
-               : walk_chunk<D, G, false, Q>(pt, q, s.p_trees, s.tree_bytes, xcol, row_bytes, 0.0f, la);
-    if (Q > 1) {
-      __syncthreads();
-      if (q == 0)
-        for (int t = 0; t < s.p_trees; ++t) accp += park[t * TC + c];
+    failed = !__syncthreads_and(mbar_wait_bounded(smem_u32(&bars[2]), 0u));
+    if (!failed) {
+      accp = nan ? walk_chunk<D, G, true, Q>(pt, q, s.p_trees, s.tree_bytes, xcol, row_bytes, 0.0f, la)
+                 : walk_chunk<D, G, false, Q>(pt, q, s.p_trees, s.tree_bytes, xcol, row_bytes, 0.0f, la);
+      if (Q > 1) {
+        __syncthreads();
+        if (q == 0)
+          for (int t = 0; t < s.p_trees; ++t) accp += park[t * TC + c];
+      }
     }
+  }
+  if (failed) {
+    if (tid == 0) {
+      // both copies land before the CTA's shared memory is released
+      mbar_wait_bounded(smem_u32(&bars[0]), 0u);
+      mbar_wait_bounded(smem_u32(&bars[2]), 0u);
+      atomicOr(s.err, kErrWaitTimeout);
+    }
+    accv = -INFINITY;  // the tile's bookkeeping still completes, none of it valid
   }
   pdl_trigger();
   if (q == 0) {  // whole warps of group 0
