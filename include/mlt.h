@@ -313,13 +313,40 @@ int mlt_decode_knobs(void *stream, const int32_t *radices, const float *option_v
                      int64_t n, uint8_t *out_knobs, float *out_feats);
 
 /* mlt_screen over decoded candidates first_index .. first_index+n-1: the
- * features are built on chip inside the screening kernels and never stored.
+ * features are built on chip inside the screening kernels and never stored
+ * (below the compiled-program threshold, see mlt_tune_decode_jit).
  * The program length must equal the current F.  out_topk holds candidate
- * indices (first_index + position).  Asynchronous on `stream`. */
+ * indices (first_index + position).  Batches of at least the
+ * mlt_tune_decode_jit threshold instead build their rows once with the
+ * compiled feature program and screen them (same results).  Asynchronous on
+ * `stream`. */
 int mlt_screen_decoded(void *stream, const int32_t *radices, const float *option_values,
                        int n_knobs, const mlt_feat_op *program, int64_t first_index,
                        int64_t n, float thr, int k, float *out_pvalid, float *out_perf,
                        int64_t *out_topk);
+
+/* Compiled feature program (no counterpart in the paper's text; an
+ * implementation choice for decoded screening).  Inside the walk kernels
+ * the feature program is interpreted one operation at a time.  For a
+ * decoded batch of at least min_n candidates (mlt_screen_decoded and the
+ * calls built on it) the library instead generates CUDA C from the program
+ * -- one statement per feature, the same correctly rounded operation as the
+ * interpreter, constants as exact bit patterns -- compiles it with NVRTC
+ * once per program and device (the first such call pays the compilation,
+ * tens to hundreds of milliseconds), runs it to write the batch's rows
+ * [n][F] into a library-owned device buffer (n x F x 4 bytes, grown as
+ * needed and kept until exit), and screens those rows.  Results are
+ * bit-identical to the interpreted path; only the time differs.  Where
+ * NVRTC (libnvrtc.so.13) or the driver library cannot be loaded, or the
+ * compilation fails, the call keeps the interpreted path.
+ *   min_n   0 (never compile) or the smallest batch that uses it; the
+ *           default is 1,048,576
+ * mlt_decode_jit_available: 1 if NVRTC and the driver library load.
+ * mlt_decode_jit_calls: screening calls so far that ran the compiled
+ * program.  Host-only. */
+int mlt_tune_decode_jit(int64_t min_n);
+int mlt_decode_jit_available(void);
+int64_t mlt_decode_jit_calls(void);
 
 /* Wait for `stream` and report errors its queued library work met on the
  * device (MLT_ETIMEOUT for a bounded wait that gave up), clearing them. */

@@ -96,6 +96,9 @@ struct ScratchOwner {
   float* sa_pvalid = nullptr;
   float* sa_perf = nullptr;
   int64_t* sa_topk = nullptr;
+  // rows of compiled-decoder batches, grown with n x F
+  float* feat_buf = nullptr;
+  long long feat_cap = 0;
   // host-buffer entry point staging
   long long host_cap_n = -1;
   int host_cap_F = 0;
@@ -135,6 +138,10 @@ ShapeOverride g_shape[3];
 // nothing completes, for g_stall_ns (one shot)
 int g_head_levels = kSplitHeadDefault;  // split tables for deep V and P models (0: compact tables)
 long long g_small_max = kSmallMaxN;     // batches up to this size screen in one launch when eligible
+// decoded batches of at least this many candidates use the compiled feature
+// program (0: never); the count of calls that did
+long long g_jit_min_n = 1LL << 20;
+long long g_jit_calls = 0;
 int g_stall_cta = -1;
 unsigned long long g_stall_ns = 0;
 
@@ -177,6 +184,27 @@ void free_model(Model& m) {
 }
 
 // Scratch sized by n candidates (plus the fixed pieces).
+// The compiled decoder's row buffer: at least `elems` floats on the scratch
+// device (grown, never shrunk; kept until exit).
+int ensure_feat_buf(long long elems) {
+  if (elems <= g_scr.feat_cap) return MLT_OK;
+  if (g_scr.feat_buf != nullptr) {
+    cudaDeviceSynchronize();
+    cudaFree(g_scr.feat_buf);
+    g_scr.feat_buf = nullptr;
+    g_scr.feat_cap = 0;
+  }
+  void* p = nullptr;
+  cudaError_t e = cudaMalloc(&p, static_cast<size_t>(elems) * sizeof(float));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(MLT_ENOMEM, "cannot allocate %lld bytes for decoded rows", elems * 4);
+  }
+  g_scr.feat_buf = static_cast<float*>(p);
+  g_scr.feat_cap = elems;
+  return MLT_OK;
+}
+
 int ensure_scratch(long long n) {
   int dev = 0;
   int rc = current_device(&dev);
@@ -462,6 +490,22 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   if (rc != MLT_OK) return rc;
   const DeviceModel& V = g_models[MLT_MODEL_V].dm;
   const DeviceModel& P = g_models[MLT_MODEL_P].dm;
+  // a large decoded batch: the compiled feature program writes its rows
+  // once, and the walks stage them like stored features (the same bits as
+  // decoding inside the walks); top-k positions stay candidate indices
+  const long long topk_base = dec ? dec->first_index : 0;
+  const DecodeParams* jit_dec = nullptr;
+  JitDecoder jd{};
+  if (dec != nullptr && g_jit_min_n > 0 && n >= g_jit_min_n) {
+    jd = jit_decoder_for(*dec, dev);
+    if (jd.fn != nullptr) {
+      rc = ensure_feat_buf(n * static_cast<long long>(g_F));
+      if (rc != MLT_OK) return rc;
+      jit_dec = dec;
+      feats = g_scr.feat_buf;
+      dec = nullptr;
+    }
+  }
   // the P pass walks the survivors; plan it for about half the batch
   const ScreenShape sv = plan_for(V, g_F, n, g_shape[MLT_MODEL_V], true);
   const ScreenShape sp = plan_for(P, g_F, (n + 1) / 2, g_shape[MLT_MODEL_P], false);
@@ -511,9 +555,14 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
     g_events_used += kPhases + 1;
     MLT_CUDA(cudaEventRecord(ev[0], st), "cudaEventRecord");
   }
+  if (jit_dec != nullptr) {  // recorded with the V phase
+    MLT_CUDA(launch_jit_decode(jd, *jit_dec, n, g_scr.feat_buf, st), "compiled decoder launch");
+    g_launches += 1;
+    g_jit_calls += 1;
+  }
   // a small batch of stored features: the whole step in one launch (its
   // time is recorded as the V phase)
-  if (dec == nullptr && n <= g_small_max) {
+  if (dec == nullptr && jit_dec == nullptr && n <= g_small_max) {
     const SmallPlan pl = plan_small(g_F, n, V, P, sm_count(), smem_optin());
     if (pl.threads > 0) {
       int stall = -1;
@@ -557,7 +606,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   MLT_CUDA(dec ? launch_traverse_dec(P, ap, *dec, sp, tiles_p, st) : launch_traverse(P, ap, sp, tiles_p, st),
            "P pass launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[3], st), "cudaEventRecord");
-  MLT_CUDA(launch_topk(s, n, k, dec ? dec->first_index : 0, out_topk, sm_count(), nullptr, st), "top-k launch");
+  MLT_CUDA(launch_topk(s, n, k, topk_base, out_topk, sm_count(), nullptr, st), "top-k launch");
   if (ev) MLT_CUDA(cudaEventRecord(ev[4], st), "cudaEventRecord");
   g_launches += (tiles_v > 0 ? 1 : 0) + (tiles_v > 0 ? 1 : 0) + (tiles_p > 0 ? 1 : 0) + 1;
   return MLT_OK;
@@ -959,6 +1008,23 @@ int mlt_load_ensemble(int model_id, const mlt_node* nodes, int n_trees, int dept
                  : pack_ensemble(nodes, n_trees, depth, g_F, packed, dm);
   if (rc != MLT_OK) return rc;
   return install_model(model_id, packed, dm);
+}
+
+int mlt_tune_decode_jit(int64_t min_n) {
+  if (min_n < 0) return fail(MLT_EINVAL, "min_n must be >= 0, got %lld", static_cast<long long>(min_n));
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_jit_min_n = min_n;
+  return MLT_OK;
+}
+
+int mlt_decode_jit_available(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  return jit_available() ? 1 : 0;
+}
+
+int64_t mlt_decode_jit_calls(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  return g_jit_calls;
 }
 
 int mlt_tune_fused_small(int max_n) {

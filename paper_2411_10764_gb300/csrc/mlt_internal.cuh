@@ -318,6 +318,19 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args,
                                 long long n_tiles, cudaStream_t st);
 cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* out_knobs,
                                float* out_feats, cudaStream_t st);
+// jit_decode.cu: the feature program compiled at run time (NVRTC) into a
+// decode kernel that writes rows [n][F]; fn is null when that is
+// unavailable (why says why)
+struct JitDecoder {
+  void* fn;
+  int tc;
+  size_t smem;
+  const char* why;
+};
+JitDecoder jit_decoder_for(const DecodeParams& d, int dev);
+bool jit_available();
+cudaError_t launch_jit_decode(const JitDecoder& jd, const DecodeParams& d, long long n, float* out,
+                              cudaStream_t st);
 
 // Launch with programmatic dependent launch allowed: the kernel may start
 // while the previous kernel on the stream finishes; it must execute

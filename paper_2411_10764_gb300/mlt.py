@@ -75,6 +75,8 @@ def lib(build_if_missing: bool = True):
             "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
             "mlt_tune_head_levels": [i32],
             "mlt_tune_fused_small": [i32],
+            "mlt_tune_decode_jit": [i64],
+            "mlt_decode_jit_available": [],
             "mlt_walk_peak": [P, i32, P, i64, i32, P, P],
             "mlt_screen_noalloc": [P, P, i64, f32, i32, P, P, P],
             "mlt_rerank": [P, P, i64, P, i32, i32, P, P],
@@ -89,6 +91,8 @@ def lib(build_if_missing: bool = True):
             fn.restype = i32
         L.mlt_kernel_launches.argtypes = []
         L.mlt_kernel_launches.restype = i64
+        L.mlt_decode_jit_calls.argtypes = []
+        L.mlt_decode_jit_calls.restype = i64
         L.mlt_last_error.argtypes = []
         L.mlt_last_error.restype = C.c_char_p
         _lib = L
@@ -433,6 +437,23 @@ def tune_fused_small(max_n: int) -> None:
     """Batches up to max_n candidates (0 .. 8192) screen in one launch when
     their models allow it; 0 turns the single-launch path off."""
     _check(lib().mlt_tune_fused_small(int(max_n)))
+
+
+def tune_decode_jit(min_n: int) -> None:
+    """Decoded batches of at least min_n candidates build their rows with
+    the feature program compiled at run time (NVRTC) and screen those; 0
+    keeps every decoded batch on the interpreted in-walk path."""
+    _check(lib().mlt_tune_decode_jit(int(min_n)))
+
+
+def decode_jit_available() -> bool:
+    """Whether NVRTC and the CUDA driver library load in this process."""
+    return bool(lib().mlt_decode_jit_available())
+
+
+def decode_jit_calls() -> int:
+    """Screening calls so far that ran the compiled feature program."""
+    return int(lib().mlt_decode_jit_calls())
 
 
 def tune_head_levels(levels: int) -> None:

@@ -199,3 +199,12 @@ def test_merge_rejects_bad_arguments():
     assert L.mlt_merge_topk(None, None, None, -1, 5, None) == -1
     assert L.mlt_merge_topk(None, None, None, 16 * 16384 + 1, 5, None) == -1
     assert L.mlt_merge_topk(None, None, None, 10, 5, None) == -1  # NULL buffers
+
+
+def test_decode_jit_tuning_and_queries():
+    with pytest.raises(mlt.MltError):
+        mlt.tune_decode_jit(-1)
+    mlt.tune_decode_jit(0)
+    mlt.tune_decode_jit(1 << 20)
+    assert isinstance(mlt.decode_jit_available(), bool)
+    assert mlt.decode_jit_calls() >= 0
