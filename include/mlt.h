@@ -328,8 +328,9 @@ int mlt_screen_decoded(void *stream, const int32_t *radices, const float *option
 /* Compiled feature program (no counterpart in the paper's text; an
  * implementation choice for decoded screening).  Inside the walk kernels
  * the feature program is interpreted one operation at a time.  For a
- * decoded batch of at least min_n candidates (mlt_screen_decoded and the
- * calls built on it) the library instead generates CUDA C from the program
+ * decoded batch of at least min_n candidates (mlt_screen_decoded, and the
+ * proposals of mlt_sa_step; mlt_screen_until_decoded keeps the interpreter)
+ * the library instead generates CUDA C from the program
  * -- one statement per feature, the same correctly rounded operation as the
  * interpreter, constants as exact bit patterns -- compiles it with NVRTC
  * once per program and device (the first such call pays the compilation,
