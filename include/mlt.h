@@ -338,8 +338,9 @@ int mlt_screen_decoded(void *stream, const int32_t *radices, const float *option
  * [n][F] into a library-owned device buffer (n x F x 4 bytes, grown as
  * needed and kept until exit), and screens those rows.  Results are
  * bit-identical to the interpreted path; only the time differs.  Where
- * NVRTC (libnvrtc.so.13) or the driver library cannot be loaded, or the
- * compilation fails, the call keeps the interpreted path.
+ * NVRTC (libnvrtc.so.13) or the driver library cannot be loaded, the
+ * compilation fails or the row buffer cannot be allocated, the call keeps
+ * the interpreted path.
  *   min_n   0 (never compile) or the smallest batch that uses it; the
  *           default is 1,048,576
  * mlt_decode_jit_available: 1 if NVRTC and the driver library load.

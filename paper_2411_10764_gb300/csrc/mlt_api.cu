@@ -185,9 +185,10 @@ void free_model(Model& m) {
 
 // Scratch sized by n candidates (plus the fixed pieces).
 // The compiled decoder's row buffer: at least `elems` floats on the scratch
-// device (grown, never shrunk; kept until exit).
-int ensure_feat_buf(long long elems) {
-  if (elems <= g_scr.feat_cap) return MLT_OK;
+// device (grown, never shrunk; kept until exit).  False when it cannot be
+// had (the caller then decodes inside the walks, which needs no buffer).
+bool try_feat_buf(long long elems) {
+  if (elems <= g_scr.feat_cap) return true;
   if (g_scr.feat_buf != nullptr) {
     cudaDeviceSynchronize();
     cudaFree(g_scr.feat_buf);
@@ -195,14 +196,13 @@ int ensure_feat_buf(long long elems) {
     g_scr.feat_cap = 0;
   }
   void* p = nullptr;
-  cudaError_t e = cudaMalloc(&p, static_cast<size_t>(elems) * sizeof(float));
-  if (e != cudaSuccess) {
-    cudaGetLastError();
-    return fail(MLT_ENOMEM, "cannot allocate %lld bytes for decoded rows", elems * 4);
+  if (cudaMalloc(&p, static_cast<size_t>(elems) * sizeof(float)) != cudaSuccess) {
+    cudaGetLastError();  // clear the allocation failure
+    return false;
   }
   g_scr.feat_buf = static_cast<float*>(p);
   g_scr.feat_cap = elems;
-  return MLT_OK;
+  return true;
 }
 
 int ensure_scratch(long long n) {
@@ -498,9 +498,7 @@ int run_screen_with(cudaStream_t st, const float* feats, const DecodeParams* dec
   JitDecoder jd{};
   if (dec != nullptr && g_jit_min_n > 0 && n >= g_jit_min_n) {
     jd = jit_decoder_for(*dec, dev);
-    if (jd.fn != nullptr) {
-      rc = ensure_feat_buf(n * static_cast<long long>(g_F));
-      if (rc != MLT_OK) return rc;
+    if (jd.fn != nullptr && try_feat_buf(n * static_cast<long long>(g_F))) {
       jit_dec = dec;
       feats = g_scr.feat_buf;
       dec = nullptr;
