@@ -537,7 +537,9 @@ def measure_workload(ctx, w, args, headline: bool):
         torch.cuda.synchronize(ctx.dev)
         est = max(e0.elapsed_time(e1), 1e-3)
         steps = int(min(20000, max(args.steps, math.ceil(MIN_TIMED_S * 1e3 / est))))
+    jit0 = mlt.decode_jit_calls()
     ms, clocks, launches, wall = timed_steps(ctx, step, steps, ctx.rank == 0)
+    jit_steps = mlt.decode_jit_calls() - jit0
     phases = phase_pass(ctx, step, min(steps, 200))
     pv, pf, tk = (bufs[k].cpu().numpy() for k in ("pv", "pf", "tk"))
     hbm_gbs, sm_max, peak_src = peaks()
@@ -588,6 +590,9 @@ def measure_workload(ctx, w, args, headline: bool):
         "gpu_launches": int(launches), "clocks": clocks,
         "wall_ms_per_step_incl_flush": wall * 1e3 / steps,
     }
+    if w.decoder is not None:
+        rec["decode_path"] = ("compiled feature program (NVRTC): rows written once per step, then screened"
+                              if jit_steps == steps else "interpreted inside the walk kernels")
     if ctx.rank == 0 and ctx.world == 1 and not args.no_cpu_baseline:
         rec["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds if headline else args.cpu_seconds_per_config)
     return rec, bufs
@@ -793,6 +798,8 @@ def run_ours(args):
     }
     if "cpu_baseline" in head:
         line["cpu_baseline"] = head["cpu_baseline"]
+    if "decode_path" in head:
+        line["decode_path"] = head["decode_path"]
     if per_config is not None:
         line["per_config"] = per_config
     if extra is not None:
