@@ -218,15 +218,16 @@ def run_reference(args):
 def walk_source_hash() -> str:
     """Hash of the sources the tree-walk kernels compile from (the walk
     device code, the launch planners and instantiations, the internal
-    header) and of the sources that decide what a step's walks read (the
-    screening sequence, the compiled feature program), in a fixed order."""
+    header, which also holds the batch size from which decoded steps use the
+    compiled feature program) and of that program's generator, in a fixed
+    order."""
     import glob
     import hashlib
 
     csrc = os.path.join(ROOT, "paper_2411_10764_gb300", "csrc")
     files = [os.path.join(csrc, "walk.cuh"), os.path.join(csrc, "mlt_internal.cuh")]
     files += sorted(glob.glob(os.path.join(csrc, "traverse*.cu")))
-    files += [os.path.join(csrc, "mlt_api.cu"), os.path.join(csrc, "jit_decode.cu")]
+    files += [os.path.join(csrc, "jit_decode.cu")]
     h = hashlib.sha256()
     for path in files:
         with open(path, "rb") as f:

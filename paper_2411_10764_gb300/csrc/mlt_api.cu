@@ -140,7 +140,7 @@ int g_head_levels = kSplitHeadDefault;  // split tables for deep V and P models 
 long long g_small_max = kSmallMaxN;     // batches up to this size screen in one launch when eligible
 // decoded batches of at least this many candidates use the compiled feature
 // program (0: never); the count of calls that did
-long long g_jit_min_n = 1LL << 20;
+long long g_jit_min_n = kDecodeJitMinN;
 long long g_jit_calls = 0;
 int g_stall_cta = -1;
 unsigned long long g_stall_ns = 0;

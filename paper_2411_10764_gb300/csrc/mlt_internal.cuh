@@ -318,6 +318,9 @@ cudaError_t launch_traverse_dec(const DeviceModel& m, const TraverseArgs& args,
                                 long long n_tiles, cudaStream_t st);
 cudaError_t launch_decode_rows(const DecodeParams& dec, long long n, uint8_t* out_knobs,
                                float* out_feats, cudaStream_t st);
+// Decoded batches of at least this many candidates build their rows with the
+// compiled feature program by default (mlt_tune_decode_jit changes it).
+constexpr long long kDecodeJitMinN = 1LL << 20;
 // jit_decode.cu: the feature program compiled at run time (NVRTC) into a
 // decode kernel that writes rows [n][F]; fn is null when that is
 // unavailable (why says why)
