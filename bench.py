@@ -571,7 +571,9 @@ def measure_workload(ctx, w, args, headline: bool):
         "roofline": {
             "bound": "alu", "kernel": f"{dominant} (tree walk)",
             "achieved": achieved / 1e9, "peak": visit_peak / 1e9, "unit": "Gvisit/s",
-            "frac": achieved / visit_peak, "traffic": dram_traffic(w.cfg.id, dominant),
+            "frac": achieved / visit_peak,
+            # the committed counters were taken at each workload's full size
+            "traffic": dram_traffic(w.cfg.id, dominant) if w.n == w.cfg.n else None,
             "peak_note": f"152 SMs x 32 shared-memory lanes/clk x {sm_max:.0f} MHz: one x[f] gather per node visit",
             "measured_walk_peak": None if ceiling is None else dict(ceiling, frac=achieved / 1e9 / ceiling["value"]),
         },
