@@ -593,6 +593,9 @@ def measure_workload(ctx, w, args, headline: bool):
         "gpu_launches": int(launches), "clocks": clocks,
         "wall_ms_per_step_incl_flush": wall * 1e3 / steps,
     }
+    rec["walk_shapes"] = {"v": mlt.walk_shape(mlt.MLT_MODEL_V, w.n), "p": mlt.walk_shape(mlt.MLT_MODEL_P, w.n, True),
+                          "note": "planned shape of each pass's walk (a step of one launch uses the single-launch "
+                                  "kernel instead)" if launches == steps else "planned shape of each pass's walk"}
     if w.decoder is not None:
         rec["decode_path"] = ("compiled feature program (NVRTC): rows written once per step, then screened"
                               if jit_steps == steps else "interpreted inside the walk kernels")
@@ -803,6 +806,7 @@ def run_ours(args):
         line["cpu_baseline"] = head["cpu_baseline"]
     if "decode_path" in head:
         line["decode_path"] = head["decode_path"]
+    line["walk_shapes"] = head["walk_shapes"]
     if per_config is not None:
         line["per_config"] = per_config
     if extra is not None:

@@ -434,6 +434,17 @@ int mlt_phase_times(float *out_ms, int n_phases, int64_t *n_calls_out);
  * choice.  Results never depend on the shape.  Host-only. */
 int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf);
 
+/* Measurement: the launch shape the tree walk over model `model_id`'s
+ * trees (V or P, loaded on the current device) would use for a screening
+ * call of n candidates -- the V pass (p_pass = 0) walks n, the P pass
+ * (p_pass != 0) is planned for about half of them -- including any shape
+ * fixed by mlt_tune_walk.  out[7]: candidates per CTA, splits (tree groups
+ * or lanes per candidate), trees in flight per thread, trees per chunk,
+ * chunk buffers, CTAs resident per SM, table kind (0 full, 1 compact,
+ * 2 half, 3 split).  Batches that mlt_screen screens in one launch
+ * (mlt_tune_fused_small) do not use this shape.  Host-only. */
+int mlt_walk_shape(int model_id, int64_t n, int p_pass, int32_t *out);
+
 /* Tuning: batches of up to max_n candidates (0 .. 8,192; the default is
  * 8,192) with stored features, whose V and P are full tables (depth <= 10)
  * of the same depth small enough to share a CTA's shared memory, are

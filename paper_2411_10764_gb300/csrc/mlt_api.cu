@@ -1559,6 +1559,31 @@ int mlt_walk_peak(void* stream, int model_id, const float* feats, int64_t n, int
   return MLT_OK;
 }
 
+int mlt_walk_shape(int model_id, int64_t n, int p_pass, int32_t* out) {
+  if (model_id != MLT_MODEL_V && model_id != MLT_MODEL_P)
+    return fail(MLT_EINVAL, "model id must be V (0) or P (1), got %d", model_id);
+  if (out == nullptr) return fail(MLT_EINVAL, "out must be non-NULL");
+  if (n < 1) return fail(MLT_EINVAL, "n must be >= 1, got %lld", static_cast<long long>(n));
+  std::lock_guard<std::mutex> lk(g_mu);
+  int dev = 0;
+  int rc = current_device(&dev);
+  if (rc != MLT_OK) return rc;
+  const Model& m = g_models[model_id];
+  if (!m.loaded) return fail(MLT_ENOMODEL, "model %d is not loaded", model_id);
+  if (m.device != dev) return fail(MLT_EINVAL, "model %d lives on device %d, current device is %d", model_id, m.device, dev);
+  // the P pass is planned for about half the batch, as the screening does
+  const ScreenShape sh = plan_for(m.dm, g_F, p_pass ? (n + 1) / 2 : n, g_shape[model_id], !p_pass);
+  if (sh.threads == 0) return fail(MLT_EINVAL, "F=%d leaves no room for a shared-memory tile", g_F);
+  out[0] = sh.threads;
+  out[1] = sh.lanes;
+  out[2] = sh.group;
+  out[3] = sh.chunk_trees;
+  out[4] = sh.nbuf;
+  out[5] = sh.resident;
+  out[6] = m.dm.kind;
+  return MLT_OK;
+}
+
 int mlt_tune_walk(int model_id, int candidates, int splits, int group, int chunk_trees, int nbuf) {
   if (model_id < MLT_MODEL_V || model_id > MLT_MODEL_A) return fail(MLT_EINVAL, "unknown model id %d", model_id);
   if (candidates < 0 || candidates > kFullMaxTile || candidates % 32 != 0)

@@ -73,6 +73,7 @@ def lib(build_if_missing: bool = True):
             "mlt_profile_phases": [i32],
             "mlt_phase_times": [P, i32, P],
             "mlt_tune_walk": [i32, i32, i32, i32, i32, i32],
+            "mlt_walk_shape": [i32, i64, i32, P],
             "mlt_tune_head_levels": [i32],
             "mlt_tune_fused_small": [i32],
             "mlt_tune_decode_jit": [i64],
@@ -437,6 +438,16 @@ def tune_fused_small(max_n: int) -> None:
     """Batches up to max_n candidates (0 .. 8192) screen in one launch when
     their models allow it; 0 turns the single-launch path off."""
     _check(lib().mlt_tune_fused_small(int(max_n)))
+
+
+def walk_shape(model_id: int, n: int, p_pass: bool = False) -> dict:
+    """The launch shape the walk over model_id's trees would use for a
+    screening call of n candidates (P pass: planned for about n/2)."""
+    out = np.zeros(7, dtype=np.int32)
+    _check(lib().mlt_walk_shape(int(model_id), int(n), 1 if p_pass else 0, out.ctypes.data))
+    kinds = {0: "full", 1: "compact", 2: "half", 3: "split"}
+    return {"candidates": int(out[0]), "splits": int(out[1]), "group": int(out[2]), "chunk_trees": int(out[3]),
+            "nbuf": int(out[4]), "resident": int(out[5]), "table": kinds.get(int(out[6]), str(int(out[6])))}
 
 
 def tune_decode_jit(min_n: int) -> None:

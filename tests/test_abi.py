@@ -208,3 +208,9 @@ def test_decode_jit_tuning_and_queries():
     mlt.tune_decode_jit(1 << 20)
     assert isinstance(mlt.decode_jit_available(), bool)
     assert mlt.decode_jit_calls() >= 0
+
+
+@pytest.mark.parametrize("args", [(2, 10, 0), (5, 10, 0), (0, 0, 0), (1, -3, 1)])
+def test_walk_shape_rejects(args):
+    with pytest.raises(mlt.MltError):
+        mlt.walk_shape(*args)

@@ -173,3 +173,26 @@ def test_full_walk_decoded_shapes(decoded, cand, splits, group, chunk):
     finally:
         _release()
     assert_parity(got, _expected("decoded", decoded))
+
+
+def test_walk_shape_reports_the_planned_and_the_forced_shape(full):
+    mlt.load_workload_models(full)
+    n = 1 << 20
+    try:
+        _force(candidates=96, splits=2, group=4, chunk_trees=8, nbuf=2)
+        for p_pass in (False, True):
+            sh = mlt.walk_shape(mlt.MLT_MODEL_V if not p_pass else mlt.MLT_MODEL_P, n, p_pass)
+            assert (sh["candidates"], sh["splits"], sh["group"], sh["chunk_trees"], sh["nbuf"]) == (96, 2, 4, 8, 2)
+            assert sh["table"] == "full"
+    finally:
+        _release()
+
+
+def test_walk_shape_of_the_decoded_conv2d_space():
+    """Depth-10 trees of 10,272 bytes beside 96 fp32 features: one CTA of 384
+    candidates per SM with two 4-tree chunks, 4 trees in flight."""
+    w = W.make_workload(4, seed=1, n=4096)
+    mlt.load_workload_models(w)
+    sh = mlt.walk_shape(mlt.MLT_MODEL_V, 1 << 24)
+    assert (sh["candidates"], sh["splits"], sh["group"], sh["chunk_trees"], sh["nbuf"], sh["resident"]) == \
+        (384, 1, 4, 4, 2, 1)
